@@ -1,0 +1,314 @@
+// Prompt-phase DMC compression (Algorithm 1 over a prompt, without attention).
+//
+// With binary alpha, Eq. partial-accumulation makes every slot the
+// omega-weighted mean of one segment of consecutive tokens: a segment opens at
+// a token with alpha = 0 (k[0] < 0) or at the first token of an empty head, and
+// runs up to the next opening token; z of the slot is the segment's summed
+// omega. Two kernels, no host synchronisation:
+//
+//  plan: one block per (sequence, KV head). Reads k[t, h, 0] of the prompt,
+//        records which tokens open a slot (one byte per token and head), counts
+//        openings per 128-token chunk, takes pages for the head's new slots from
+//        the pool (one atomic per head), and stores each chunk's first slot index.
+//  scan: one block per (128-token chunk, KV head, sequence). The block owns the
+//        segments that open inside its chunk (and chunk 0 also owns the tokens
+//        that continue the head's existing last slot); a segment that runs past
+//        the chunk end is followed to its end, so each k/v row is read once.
+//        Warps take segments round-robin; lanes split a row into 16-byte pieces
+//        and accumulate sum(omega k), sum(omega v), sum(omega) in fp32; the slot
+//        is the quotient, rounded once to the cache dtype.
+#include "dmc_internal.cuh"
+
+namespace dmc {
+
+constexpr int kPlanThreads = 256;
+constexpr int kScanThreads = 128;
+
+struct PrefillArgs {
+  Layout lay;
+  int layer, first_seq, num_seqs;
+  const char* q;
+  long long q_tok, q_head;  // element strides of the queries' first components
+  const char* k;
+  const char* v;
+  const int* cu;
+  int total_tokens, max_seqlen;
+};
+
+__device__ __forceinline__ bool seq_bounds(const PrefillArgs& a, int s, int& t0, int& t1) {
+  t0 = a.cu[s];
+  t1 = a.cu[s + 1];
+  return t0 >= 0 && t0 <= t1 && t1 <= a.total_tokens && (t1 - t0) <= a.max_seqlen;
+}
+
+__device__ __forceinline__ int chunk_id(int t0, int c, int s) { return (t0 + c * kPrefillChunk) / kPrefillChunk + s; }
+
+template <typename T, int D>
+__global__ void __launch_bounds__(kPlanThreads) dmc_prefill_plan_kernel(const PrefillArgs a) {
+  extern __shared__ int cnt[];  // [ceil(max_seqlen / 128)]
+  __shared__ int s_fail, s_first_page, s_nan, s_wsum[kPlanThreads / 32 + 1];
+  const Layout& L = a.lay;
+  const int s = blockIdx.x, h = blockIdx.y;
+  const int bh = (a.first_seq + s) * L.Hkv + h;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int parity = *reinterpret_cast<volatile int*>(&L.ctl[a.layer * 4]);
+  int* len = L.lengths + ((size_t)a.layer * 2 + parity) * L.NH;
+  int t0, t1;
+  if (!seq_bounds(a, s, t0, t1)) {
+    if (tid == 0) atomicOr(L.error, DMC_FAULT_BAD_SEQLENS);
+    return;
+  }
+  const int ntok = t1 - t0;
+  const int nch = ceil_div(ntok, kPrefillChunk);
+  const int len_old = len[bh];
+  for (int c = tid; c < nch; c += kPlanThreads) cnt[c] = 0;
+  if (tid == 0) { s_fail = 0; s_nan = 0; }
+  __syncthreads();
+  const T* kk = reinterpret_cast<const T*>(a.k);
+  for (int base = 0; base < ntok; base += kPlanThreads) {
+    const int i = base + tid;
+    bool opens = false;
+    if (i < ntok) {
+      const size_t t = (size_t)(t0 + i);
+      const float x = Elt<T>::to_f(kk[(t * L.Hkv + h) * D]);
+      if (x != x) s_nan = 1;
+      // alpha = round(sigmoid(k[0])) = [k[0] >= 0]; alpha = 0 opens a slot,
+      // and so does the first token of an empty head.
+      opens = !(x >= 0.f) || (i == 0 && len_old == 0);
+      L.opens[t * L.Hkv + h] = opens ? 1 : 0;
+    }
+    const unsigned bal = __ballot_sync(0xffffffffu, opens);
+    if (lane == 0 && base + warp * 32 < ntok) atomicAdd(&cnt[(base + warp * 32) / kPrefillChunk], __popc(bal));
+  }
+  __syncthreads();
+  // exclusive scan of the chunk counts (nch <= max_seqlen / 128 + 1)
+  const int per = ceil_div(nch, kPlanThreads);
+  const int c0 = min(tid * per, nch), c1 = min(c0 + per, nch);
+  int local = 0;
+  for (int c = c0; c < c1; ++c) local += cnt[c];
+  int incl = local;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const int o = __shfl_up_sync(0xffffffffu, incl, off);
+    if (lane >= off) incl += o;
+  }
+  if (lane == 31) s_wsum[warp] = incl;
+  __syncthreads();
+  if (tid == 0) {
+    int run = 0;
+    for (int w = 0; w < kPlanThreads / 32; ++w) { const int t = s_wsum[w]; s_wsum[w] = run; run += t; }
+    s_wsum[kPlanThreads / 32] = run;
+  }
+  __syncthreads();
+  const int new_slots = s_wsum[kPlanThreads / 32];
+  const int len_new = len_old + new_slots;
+  const int old_pages = ceil_div(len_old, kPage), new_pages = ceil_div(len_new, kPage);
+  const int need = new_pages - old_pages;
+  if (tid == 0) {
+    int fail = 0, first = 0;
+    if (len_new > L.max_slots) {
+      atomicOr(L.error, DMC_FAULT_SLOT_CAPACITY);
+      fail = 1;
+    } else if (need > 0) {
+      const unsigned long long f = atomicAdd(L.pool_top, (unsigned long long)need);
+      if (f + (unsigned long long)need > (unsigned long long)L.num_pages) {
+        atomicOr(L.error, DMC_FAULT_PAGES_EXHAUSTED);
+        fail = 1;
+      } else {
+        first = (int)f;
+      }
+    }
+    if (s_nan) atomicOr(L.error, DMC_FAULT_NAN_GATE);
+    s_fail = fail;
+    s_first_page = first;
+  }
+  __syncthreads();
+  const int fail = s_fail;
+  int run = s_wsum[warp] + incl - local;
+  for (int c = c0; c < c1; ++c) {
+    L.plan[(size_t)h * L.plan_stride + chunk_id(t0, c, s)] = fail ? -1 : len_old + run;
+    run += cnt[c];
+  }
+  if (!fail) {
+    int* pt = L.page_table + ((size_t)a.layer * L.NH + bh) * L.MPH;
+    for (int i = tid; i < need; i += kPlanThreads) pt[old_pages + i] = s_first_page + i;
+    if (tid == 0) len[bh] = len_new;
+  }
+}
+
+template <typename T, int D>
+__device__ __forceinline__ void scan_segment(const PrefillArgs& a, int h, int bh, int tb, int te,
+                                             int slot, bool merge_old) {
+  using CK = Chunk<T>;
+  constexpr int ROW = D * (int)sizeof(T);
+  constexpr int LPR = ROW / 16;  // lanes per row
+  constexpr int RPI = 32 / LPR;  // rows per warp iteration
+  constexpr int EPC = CK::N;
+  const Layout& L = a.lay;
+  const int lane = threadIdx.x & 31, sub = lane / LPR, lr = lane % LPR;
+  const T* qq = reinterpret_cast<const T*>(a.q);
+  float ak[EPC], av[EPC], zs = 0.f;
+#pragma unroll
+  for (int e = 0; e < EPC; ++e) { ak[e] = 0.f; av[e] = 0.f; }
+  const size_t hrow = (size_t)L.Hkv * ROW;
+  const char* kb = a.k + (size_t)h * ROW + lr * 16;
+  const char* vb = a.v + (size_t)h * ROW + lr * 16;
+#pragma unroll 2
+  for (int t = tb + sub; t < te; t += RPI) {
+    const uint4 kr = __ldg(reinterpret_cast<const uint4*>(kb + (size_t)t * hrow));
+    const uint4 vr = __ldg(reinterpret_cast<const uint4*>(vb + (size_t)t * hrow));
+    float y = 0.f;
+    for (int g = 0; g < L.G; ++g)
+      y += Elt<T>::to_f(qq[(size_t)t * a.q_tok + (size_t)(h * L.G + g) * a.q_head]);
+    const float w = sigmoidf_(y / (float)L.G);  // omega = sigmoid(q[0]) (group mean for GQA)
+    float kf[EPC], vf[EPC];
+    CK::unpack(kr, kf);
+    CK::unpack(vr, vf);
+    if (lr == 0) kf[0] = 0.f;  // k[0] <- 0 (Algorithm 1)
+#pragma unroll
+    for (int e = 0; e < EPC; ++e) {
+      ak[e] = fmaf(w, kf[e], ak[e]);
+      av[e] = fmaf(w, vf[e], av[e]);
+    }
+    zs += w;
+  }
+#pragma unroll
+  for (int off = LPR; off < 32; off <<= 1) {
+#pragma unroll
+    for (int e = 0; e < EPC; ++e) {
+      ak[e] += __shfl_xor_sync(0xffffffffu, ak[e], off);
+      av[e] += __shfl_xor_sync(0xffffffffu, av[e], off);
+    }
+    zs += __shfl_xor_sync(0xffffffffu, zs, off);
+  }
+  if (sub != 0) return;
+  const int page = L.page_table[((size_t)a.layer * L.NH + bh) * L.MPH + slot / kPage];
+  char* kdst = L.pages + (size_t)page * L.page_bytes + (size_t)(slot % kPage) * ROW + lr * 16;
+  char* vdst = kdst + (size_t)kPage * ROW;
+  float* zp = L.z + (size_t)page * kPage + slot % kPage;
+  float kn[EPC], vn[EPC], znew;
+  if (merge_old) {
+    // the prompt continues the head's last slot: (K z_old + sum w k) / (z_old + sum w)
+    float ko[EPC], vo[EPC];
+    CK::unpack(*reinterpret_cast<const uint4*>(kdst), ko);
+    CK::unpack(*reinterpret_cast<const uint4*>(vdst), vo);
+    const float zo = *zp;
+    znew = zo + zs;
+#pragma unroll
+    for (int e = 0; e < EPC; ++e) {
+      kn[e] = (ko[e] * zo + ak[e]) / znew;
+      vn[e] = (vo[e] * zo + av[e]) / znew;
+    }
+  } else {
+    znew = zs;
+#pragma unroll
+    for (int e = 0; e < EPC; ++e) {
+      kn[e] = ak[e] / zs;
+      vn[e] = av[e] / zs;
+    }
+  }
+  if (lr == 0) kn[0] = 0.f;
+  *reinterpret_cast<uint4*>(kdst) = CK::pack(kn);
+  *reinterpret_cast<uint4*>(vdst) = CK::pack(vn);
+  if (lr == 0) *zp = znew;
+}
+
+template <typename T, int D>
+__global__ void __launch_bounds__(kScanThreads) dmc_prefill_scan_kernel(const PrefillArgs a) {
+  __shared__ int starts[kPrefillChunk];
+  __shared__ int s_wcnt[kScanThreads / 32];
+  __shared__ int s_next;
+  const Layout& L = a.lay;
+  const int c = blockIdx.x, h = blockIdx.y, s = blockIdx.z;
+  const int bh = (a.first_seq + s) * L.Hkv + h;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  int t0, t1;
+  if (!seq_bounds(a, s, t0, t1)) return;
+  const int a0 = t0 + c * kPrefillChunk;
+  if (a0 >= t1) return;
+  const int a1 = min(a0 + kPrefillChunk, t1);
+  const int base = L.plan[(size_t)h * L.plan_stride + chunk_id(t0, c, s)];
+  if (base < 0) return;
+  const unsigned char* op = L.opens + h;
+  const size_t ostride = (size_t)L.Hkv;
+
+  // positions of the tokens of [a0, a1) that open a slot, in order
+  static_assert(kScanThreads == kPrefillChunk, "one thread per chunk token");
+  const int t = a0 + tid;
+  const bool f = (t < a1) && op[(size_t)t * ostride];
+  const unsigned bal = __ballot_sync(0xffffffffu, f);
+  if (lane == 0) s_wcnt[warp] = __popc(bal);
+  if (tid == 0) s_next = t1;
+  __syncthreads();
+  int before = __popc(bal & ((1u << lane) - 1u));
+  for (int w = 0; w < warp; ++w) before += s_wcnt[w];
+  int nstart = 0;
+  for (int w = 0; w < kScanThreads / 32; ++w) nstart += s_wcnt[w];
+  if (f) starts[before] = t;
+  // the first opening token at or after a1 ends the chunk's last segment
+  for (int b0 = a1; b0 < t1; b0 += kScanThreads) {
+    const int tt = b0 + tid;
+    const bool g = tt < t1 && op[(size_t)tt * ostride];
+    if (g) atomicMin(&s_next, tt);
+    if (__syncthreads_or(g)) break;
+  }
+  __syncthreads();
+  const int next = s_next;
+  const bool pre = (c == 0) && !op[(size_t)t0 * ostride];  // continues the existing last slot
+  const int items = nstart + (pre ? 1 : 0);
+  for (int it = warp; it < items; it += kScanThreads / 32) {
+    if (pre && it == 0) {
+      const int te = nstart > 0 ? starts[0] : next;
+      scan_segment<T, D>(a, h, bh, t0, te, base - 1, true);
+    } else {
+      const int j = it - (pre ? 1 : 0);
+      const int tb = starts[j];
+      const int te = (j + 1 < nstart) ? starts[j + 1] : next;
+      scan_segment<T, D>(a, h, bh, tb, te, base + j, false);
+    }
+  }
+}
+
+template <typename T, int D>
+static cudaError_t launch_prefill(const PrefillArgs& a, cudaStream_t stream) {
+  const int max_chunks = ceil_div(a.max_seqlen, kPrefillChunk);
+  const size_t plan_smem = (size_t)max(max_chunks, 1) * sizeof(int);
+  if (plan_smem > 48 * 1024) {
+    cudaError_t e = cudaFuncSetAttribute(dmc_prefill_plan_kernel<T, D>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)plan_smem);
+    if (e != cudaSuccess) return e;
+  }
+  dmc_prefill_plan_kernel<T, D><<<dim3(a.num_seqs, a.lay.Hkv), kPlanThreads, plan_smem, stream>>>(a);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  if (max_chunks > 0) {
+    dmc_prefill_scan_kernel<T, D><<<dim3(max_chunks, a.lay.Hkv, a.num_seqs), kScanThreads, 0, stream>>>(a);
+    e = cudaGetLastError();
+  }
+  return e;
+}
+
+cudaError_t prefill_launch(const Layout& L, int layer, int first_seq, int num_seqs, const void* q,
+                           long long q_tok, long long q_head, const void* k, const void* v,
+                           const int* cu, int total_tokens, int max_seqlen, cudaStream_t stream) {
+  PrefillArgs a;
+  a.lay = L;
+  a.layer = layer;
+  a.first_seq = first_seq;
+  a.num_seqs = num_seqs;
+  a.q = static_cast<const char*>(q);
+  a.q_tok = q_tok;
+  a.q_head = q_head;
+  a.k = static_cast<const char*>(k);
+  a.v = static_cast<const char*>(v);
+  a.cu = cu;
+  a.total_tokens = total_tokens;
+  a.max_seqlen = max_seqlen;
+  if (L.esize == 4 && L.D == 64) return launch_prefill<float, 64>(a, stream);
+  if (L.esize == 4 && L.D == 128) return launch_prefill<float, 128>(a, stream);
+  if (L.esize == 2 && L.D == 64) return launch_prefill<__nv_bfloat16, 64>(a, stream);
+  if (L.esize == 2 && L.D == 128) return launch_prefill<__nv_bfloat16, 128>(a, stream);
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace dmc

@@ -1,0 +1,190 @@
+"""Helpers for the GPU parity tests: drive the CUDA path through the C ABI and
+the fp64 oracle on the same seeded inputs, and compare."""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+from oracle import cref
+from oracle import dmc_ref as R
+from paper_2403_09636_gb300 import DmcCache, synthetic as S
+
+TOL = {"f32": 1e-4, "bf16": 2e-2}
+
+
+def expected_prompt_lengths(k0_np, cu, start=None):
+    """Slot count per (sequence, head) after a prompt, from the oracle's
+    decision rule: an empty head's first token opens slot 0, and every later
+    token with alpha = 0 opens another."""
+    B = len(cu) - 1
+    H = k0_np.shape[1]
+    out = np.zeros((B, H), dtype=np.int64)
+    for b in range(B):
+        seg = k0_np[cu[b]:cu[b + 1]]
+        alpha = R.decision(seg)
+        opens = (alpha == 0).astype(np.int64)
+        s0 = np.zeros(H, dtype=np.int64) if start is None else np.asarray(start[b], dtype=np.int64)
+        if seg.shape[0]:
+            opens[0] = np.where(s0 == 0, 1, opens[0])
+        out[b] = s0 + opens.sum(axis=0)
+    return out
+
+
+def expected_step_lengths(prev, k0_np):
+    """Lengths after one decode token per head (prev [B, H], k0 [B, H])."""
+    alpha = R.decision(k0_np)
+    return prev + np.where((prev == 0) | (alpha == 0), 1, 0)
+
+
+def cache_for(wl: S.Workload, device, max_slots=None, num_pages=None, max_prefill_tokens=None):
+    lens = S.prompt_lengths(wl)
+    if max_slots is None:
+        max_slots = int(lens.max()) + wl.decode_steps + 1
+    NH = wl.batch * wl.num_kv_heads
+    if num_pages is None:
+        num_pages = wl.num_layers * NH * ((max_slots + 31) // 32)
+    if max_prefill_tokens is None:
+        max_prefill_tokens = int(lens.sum())
+    return DmcCache(wl.num_layers, wl.batch, wl.num_q_heads, wl.num_kv_heads, wl.head_dim,
+                    wl.torch_dtype, max_slots, num_pages, max_prefill_tokens, device=device)
+
+
+class Run:
+    """Prefill + decode of a workload on the GPU, keeping host copies of the
+    inputs of sampled (layer, seq, kv_head) instances and the GPU results for
+    them."""
+
+    def __init__(self, wl: S.Workload, device, samples, decode_steps=None, cache=None,
+                 check_all_lengths=True):
+        self.wl = wl
+        self.samples = list(samples)
+        G, d = wl.group, wl.head_dim
+        steps = wl.decode_steps if decode_steps is None else decode_steps
+        self.cache = cache if cache is not None else cache_for(wl, device)
+        p = S.append_prob(wl)
+        self.inst = {s: {"k_prompt": None, "k_dec": [], "v_dec": [], "q_dec": [], "out": []}
+                     for s in self.samples}
+        self.len_ok = True
+        self.len_msgs = []
+        layers = sorted({l for (l, _, _) in self.samples}) if not check_all_lengths else \
+            list(range(wl.num_layers))
+        lens_now = {}
+        for layer in range(wl.num_layers):
+            pr = S.gen_prompt(wl, layer, device, p=p)
+            self.cache.prefill(layer, pr["q0"], pr["k"], pr["v"], pr["cu_seqlens"],
+                               pr["max_seqlen"])
+            cu = pr["cu_seqlens"].cpu().numpy()
+            if layer in layers:
+                k0 = pr["k"][:, :, 0].float().cpu().numpy()
+                exp = expected_prompt_lengths(k0, cu)
+                got = self.cache.lengths(layer).cpu().numpy()
+                if not np.array_equal(exp, got):
+                    self.len_ok = False
+                    self.len_msgs.append(f"prefill layer {layer}: {np.argwhere(exp != got)[:5]}")
+                lens_now[layer] = exp
+            for s in self.samples:
+                if s[0] != layer:
+                    continue
+                _, b, h = s
+                sl = slice(int(cu[b]), int(cu[b + 1]))
+                self.inst[s]["k_prompt"] = pr["k"][sl, h].float().cpu().numpy()
+                self.inst[s]["v_prompt"] = pr["v"][sl, h].float().cpu().numpy()
+                self.inst[s]["q0_prompt"] = pr["q0"][sl, h * G:(h + 1) * G].float().cpu().numpy()
+            del pr
+        self.prompt_export = {}
+        for s in self.samples:
+            layer, b, h = s
+            k, v, z, ln = self.cache.export_heads(layer, [b * wl.num_kv_heads + h],
+                                                  int(S.prompt_lengths(wl)[b]) + 1)
+            n = int(ln[0])
+            self.prompt_export[s] = (k[0, :n].float().cpu().numpy(), v[0, :n].float().cpu().numpy(),
+                                     z[0, :n].cpu().numpy(), n)
+        Hq = wl.num_q_heads
+        for step in range(steps):
+            for layer in range(wl.num_layers):
+                dd = S.gen_decode(wl, layer, step, device, p=p)
+                out = torch.empty_like(dd["q"])
+                self.cache.decode(layer, dd["q"], dd["k"], dd["v"], out)
+                if layer in lens_now:
+                    exp = expected_step_lengths(lens_now[layer], dd["k"][:, :, 0].float().cpu().numpy())
+                    got = self.cache.lengths(layer).cpu().numpy()
+                    if not np.array_equal(exp, got):
+                        self.len_ok = False
+                        self.len_msgs.append(f"step {step} layer {layer}: {np.argwhere(exp != got)[:5]}")
+                    lens_now[layer] = exp
+                for s in self.samples:
+                    if s[0] != layer:
+                        continue
+                    _, b, h = s
+                    I = self.inst[s]
+                    I["k_dec"].append(dd["k"][b, h].float().cpu().numpy())
+                    I["v_dec"].append(dd["v"][b, h].float().cpu().numpy())
+                    I["q_dec"].append(dd["q"][b, h * G:(h + 1) * G].float().cpu().numpy())
+                    I["out"].append(out[b, h * G:(h + 1) * G].float().cpu().numpy())
+        self.final_export = {}
+        for s in self.samples:
+            layer, b, h = s
+            cap = int(S.prompt_lengths(wl)[b]) + steps + 1
+            k, v, z, ln = self.cache.export_heads(layer, [b * wl.num_kv_heads + h], cap)
+            n = int(ln[0])
+            self.final_export[s] = (k[0, :n].float().cpu().numpy(), v[0, :n].float().cpu().numpy(),
+                                    z[0, :n].cpu().numpy(), n)
+        self.status = self.cache.status()
+        self.steps = steps
+
+    def oracle(self, threads=8):
+        heads = []
+        d, G = self.wl.head_dim, self.wl.group
+        for s in self.samples:
+            I = self.inst[s]
+            heads.append({
+                "k_prompt": I["k_prompt"], "v_prompt": I["v_prompt"], "q0_prompt": I["q0_prompt"],
+                "k_dec": np.array(I["k_dec"]).reshape(-1, d), "v_dec": np.array(I["v_dec"]).reshape(-1, d),
+                "q_dec": np.array(I["q_dec"]).reshape(-1, G, d)})
+        return dict(zip(self.samples, cref.run_heads(heads, threads=threads)))
+
+    def compare(self, tol=None):
+        """Returns a list of failure strings (empty = parity)."""
+        tol = TOL[self.wl.dtype] if tol is None else tol
+        bad = list(self.len_msgs)
+        if self.status[0] != 0:
+            bad.append(f"device status {self.status}")
+        ref = self.oracle()
+        for s in self.samples:
+            r = ref[s]
+            k, v, z, n = self.prompt_export[s]
+            if n != r["prompt_len"]:
+                bad.append(f"{s} prompt len {n} != {r['prompt_len']}")
+            else:
+                for name, a, b in (("K", k, r["prompt_K"]), ("V", v, r["prompt_V"]), ("z", z, r["prompt_z"])):
+                    err = float(np.max(np.abs(a - b))) if n else 0.0
+                    if not err <= tol:
+                        bad.append(f"{s} prompt {name} max err {err}")
+            if self.steps:
+                out = np.array(self.inst[s]["out"])
+                err = float(np.max(np.abs(out - r["out"])))
+                if not err <= tol:
+                    bad.append(f"{s} decode out max err {err}")
+            k, v, z, n = self.final_export[s]
+            if n != r["len"]:
+                bad.append(f"{s} final len {n} != {r['len']}")
+            else:
+                for name, a, b in (("K", k, r["K"]), ("V", v, r["V"]), ("z", z, r["z"])):
+                    err = float(np.max(np.abs(a - b)))
+                    if not err <= tol:
+                        bad.append(f"{s} final {name} max err {err}")
+        return bad
+
+
+def all_samples(wl: S.Workload):
+    return [(l, b, h) for l in range(wl.num_layers) for b in range(wl.batch)
+            for h in range(wl.num_kv_heads)]
+
+
+def random_samples(wl: S.Workload, n, seed=0):
+    rng = np.random.default_rng(seed)
+    got = set()
+    while len(got) < n:
+        got.add((int(rng.integers(wl.num_layers)), int(rng.integers(wl.batch)),
+                 int(rng.integers(wl.num_kv_heads))))
+    return sorted(got)

@@ -1,0 +1,63 @@
+"""CUDA path vs the fp64 oracle on seeded synthetic workloads (GPU).
+
+Lengths are compared for every head of every checked layer after the prompt
+and after every decode step (bit-exact); slots, z and attention outputs of the
+sampled heads are compared element by element within the tolerance of the
+dtype: max-abs 1e-4 for fp32 caches, 2e-2 for bf16 caches (bf16 storage of a
+running mean rounds the slot at every merge; the oracle never rounds).
+"""
+import pytest
+
+from paper_2403_09636_gb300 import synthetic as S
+from tests import dmc_harness as H
+
+pytestmark = pytest.mark.gpu
+
+
+def _check(run):
+    assert run.len_ok, run.len_msgs[:5]
+    bad = run.compare()
+    assert not bad, bad[:10]
+
+
+def test_tiny_f32_every_head(cuda_dev):
+    wl = S.WORKLOADS["tiny_f32"]
+    _check(H.Run(wl, cuda_dev, H.all_samples(wl)))
+
+
+def test_mha_bf16_mixed_cr_ragged_tail(cuda_dev):
+    # 7B head shape, mixed per-head CR, prompt 300 (not a multiple of 32 or 128)
+    wl = S.shrink(S.WORKLOADS["llama2_7b_mixed"], num_layers=2, batch=4, num_q_heads=8,
+                  num_kv_heads=8, prompt=(300, 300), decode_steps=40)
+    _check(H.Run(wl, cuda_dev, H.random_samples(wl, 24, seed=1)))
+
+
+def test_mha_bf16_long_ragged_heavy_tail(cuda_dev):
+    wl = S.shrink(S.WORKLOADS["long_ragged"], num_layers=1, batch=3, num_q_heads=4,
+                  num_kv_heads=4, prompt=(100, 3000), decode_steps=16)
+    _check(H.Run(wl, cuda_dev, H.all_samples(wl)))
+
+
+def test_gqa_bf16_group8(cuda_dev):
+    wl = S.shrink(S.WORKLOADS["llama2_70b_gqa_2x"], num_layers=1, batch=3, num_q_heads=16,
+                  num_kv_heads=2, prompt=(200, 200), decode_steps=20)
+    _check(H.Run(wl, cuda_dev, H.all_samples(wl)))
+
+
+def test_bf16_head_dim_64(cuda_dev):
+    wl = S.Workload("bf16_d64", 1, 2, 6, 6, 64, "bf16", (150, 420), 24, ("choice", (1.0, 3.0, 8.0)), 0.5, seed=3)
+    _check(H.Run(wl, cuda_dev, H.all_samples(wl)))
+
+
+def test_f32_head_dim_128(cuda_dev):
+    wl = S.Workload("f32_d128", 1, 2, 4, 2, 128, "f32", (90, 130), 24, ("fixed", 3.0), 1.0, seed=4)
+    _check(H.Run(wl, cuda_dev, H.all_samples(wl)))
+
+
+def test_llama2_7b_4x_full_shape_sampled(cuda_dev):
+    """The benchmark workload itself (32 layers, batch 32, 32 heads, d 128,
+    prompt 2048, uniform 4x), lengths of every head of every layer after the
+    prompt and every decode step, slots and outputs of sampled heads. Decode
+    runs 64 of the 512 steps to keep the test short."""
+    wl = S.WORKLOADS["llama2_7b_4x"]
+    _check(H.Run(wl, cuda_dev, H.random_samples(wl, 48, seed=7), decode_steps=64))
