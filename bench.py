@@ -53,6 +53,8 @@ def parse():
     ap.add_argument("--workload", default="llama2_7b_4x")
     ap.add_argument("--decode-steps", type=int, default=None,
                     help="override the workload's decode steps (not for reported numbers)")
+    ap.add_argument("--layers", type=int, default=None,
+                    help="override the workload's layer count (small ncu cases, not for reported numbers)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -214,6 +216,8 @@ def run_ours(args, rank, world, dist):
     B.build()
     L_ = P.lib()
     wl = S.WORKLOADS[args.workload]
+    if args.layers is not None:
+        wl = S.shrink(wl, num_layers=args.layers)
     steps_dec = wl.decode_steps if args.decode_steps is None else args.decode_steps
     Lr, Bt, Hq, Hk, D = wl.num_layers, wl.batch, wl.num_q_heads, wl.num_kv_heads, wl.head_dim
     dt = wl.torch_dtype
@@ -249,8 +253,14 @@ def run_ours(args, rank, world, dist):
     before = plen[None] + torch.cumsum(app, 0) - app                     # len_old per decode step
     final = plen + app.sum(0)
     slots_read = int(before.sum())
-    pages_needed = int(((final + 31) // 32).sum())
-    max_slots = int(final.max()) + 1
+    # the e2e leg reuses layer 0's prompt for every layer and a ring of decode
+    # steps, so it needs its own page count; size the pool for both
+    ring = min(16, steps_dec)
+    app_ring = app[:ring]
+    reps = torch.tensor([(steps_dec - r + ring - 1) // ring for r in range(ring)], device=dev)
+    final_e2e = plen[0][None] + (app_ring * reps[:, None, None, None]).sum(0)
+    pages_needed = max(int(((final + 31) // 32).sum()), int(((final_e2e + 31) // 32).sum()))
+    max_slots = int(S.prompt_lengths(wl).max()) + steps_dec + 1
     max_prompt = max(pr["max_seqlen"] for pr in prompts)
     total_prompt = max(int(pr["cu_seqlens"][-1]) for pr in prompts)
     cache = P.DmcCache(Lr, Bt, Hq, Hk, D, dt, max_slots, pages_needed + 64, total_prompt, device=dev)
@@ -382,7 +392,7 @@ def run_e2e(args, wl, cache, prompts, qd, kd, vd, outs, steps_dec, dev, stream, 
     import torch
 
     Lr = wl.num_layers
-    ring = min(16, steps_dec)
+    ring = min(16, steps_dec)  # must match the pool sizing in run_ours
     pr0 = prompts[0]
     hq0 = pr0["q0"].cpu().pin_memory()
     hk = pr0["k"].cpu().pin_memory()
@@ -439,9 +449,9 @@ def run_e2e(args, wl, cache, prompts, qd, kd, vd, outs, steps_dec, dev, stream, 
         t = torch.tensor([ms], device=dev, dtype=torch.float64)
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         ms = t.item()
-    st = cache.status()[0]
+    st, bits, _ = cache.status()
     if st != 0:
-        raise RuntimeError(f"device fault in e2e: {st}")
+        raise RuntimeError(f"device fault in e2e: status {st} bits {bits:#x}")
     return {"value": world * args.steps * wl.batch * steps_dec / (ms / 1e3), "unit": "tokens/s",
             "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
             "note": f"pinned host inputs: one layer's prompt reused for all {Lr} layers, a ring of "
