@@ -131,6 +131,27 @@ dmc_status dmc_decode_step(dmc_cache_t cache, int32_t layer, const void* q_dev,
                            const void* k_dev, const void* v_dev, void* out_dev,
                            cudaStream_t stream);
 
+/* dmc_decode_step with its scratch in the library's own static device memory.
+ * The paper has no counterpart; this exists for callers that cannot allocate
+ * device memory of their own: a plugin or custom operator that a host
+ * framework hands only its input and output buffers (the framework owns every
+ * allocation), or a latency-critical loop that must not pay cudaMalloc's
+ * implicit device synchronisation. Same arguments, semantics and results as
+ * dmc_decode_step; it allocates nothing and calls no allocating routine.
+ * The scratch is the split-K partial softmax states of one launch, kept in a
+ * file-scope __device__ array of 1.04 MB (2 states of head_dim + 2 floats for
+ * each of at most 1024 blocks) that every GPU loading the library holds until
+ * the process exits; a cache whose decode grid would need more returns
+ * DMC_ERR_INVALID_ARG. Nothing in it needs to start at zero: each launch writes
+ * every state before reading it. The first call on a device looks up the
+ * array's device address on that device (which must be current and be the
+ * cache's device); make that first call before any stream capture. All calls
+ * share the one array, so calls whose launches overlap on the GPU (any caches,
+ * any streams) race and must be ordered by the caller. */
+dmc_status dmc_decode_step_static_scratch(dmc_cache_t cache, int32_t layer, const void* q_dev,
+                                          const void* k_dev, const void* v_dev, void* out_dev,
+                                          cudaStream_t stream);
+
 /* Copies the slot count of every head of `layer`, int32 [batch, num_kv_heads],
  * into out_dev (asynchronous). */
 dmc_status dmc_cache_lengths(dmc_cache_t cache, int32_t layer, int32_t* out_dev,

@@ -30,7 +30,8 @@ DMC_FAULT_WAIT_TIMEOUT = 0x10
 PAGE_SIZE = 32
 
 EXPORTED = ("dmc_cache_required_bytes", "dmc_cache_create", "dmc_cache_destroy",
-            "dmc_cache_reset", "dmc_prefill_compress", "dmc_decode_step", "dmc_cache_lengths",
+            "dmc_cache_reset", "dmc_prefill_compress", "dmc_decode_step",
+            "dmc_decode_step_static_scratch", "dmc_cache_lengths",
             "dmc_cache_export_heads", "dmc_cache_status", "dmc_status_string")
 
 
@@ -70,6 +71,7 @@ def lib():
             "dmc_prefill_compress": (C.c_int, [vp, i32, i32, i32, vp, i64, i64, vp, vp, vp, i32,
                                                i32, vp]),
             "dmc_decode_step": (C.c_int, [vp, i32, vp, vp, vp, vp, vp]),
+            "dmc_decode_step_static_scratch": (C.c_int, [vp, i32, vp, vp, vp, vp, vp]),
             "dmc_cache_lengths": (C.c_int, [vp, i32, vp, vp]),
             "dmc_cache_export_heads": (C.c_int, [vp, i32, i32, vp, i32, vp, vp, vp, vp, vp]),
             "dmc_cache_status": (C.c_int, [vp, vp, C.POINTER(C.c_uint32), C.POINTER(i64)]),
@@ -113,6 +115,12 @@ def dmc_prefill_compress(handle, layer, first_seq, num_seqs, q_ptr, q_token_stri
 
 def dmc_decode_step(handle, layer, q_ptr, k_ptr, v_ptr, out_ptr, stream) -> int:
     return lib().dmc_decode_step(handle, layer, q_ptr, k_ptr, v_ptr, out_ptr, stream)
+
+
+def dmc_decode_step_static_scratch(handle, layer, q_ptr, k_ptr, v_ptr, out_ptr, stream) -> int:
+    """dmc_decode_step for callers that cannot allocate device memory: its
+    scratch lives in the library's static device array (see include/dmc.h)."""
+    return lib().dmc_decode_step_static_scratch(handle, layer, q_ptr, k_ptr, v_ptr, out_ptr, stream)
 
 
 def dmc_cache_lengths(handle, layer, out_ptr, stream) -> int:

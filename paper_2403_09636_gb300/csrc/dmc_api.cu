@@ -16,6 +16,7 @@ cudaError_t decode_launch(const Layout& L, int layer, int Gv, int grid, size_t s
 cudaError_t prefill_launch(const Layout& L, int layer, int first_seq, int num_seqs, const void* q,
                            long long q_tok, long long q_head, const void* k, const void* v,
                            const int* cu, int total_tokens, int max_seqlen, cudaStream_t stream);
+cudaError_t decode_static_partials(int device, float** ptr, size_t* floats);
 constexpr int kMaxPartialBlocks = 1024;  // upper bound of the decode grid
 }  // namespace dmc
 
@@ -229,6 +230,31 @@ dmc_status dmc_decode_step(dmc_cache_t c, int32_t layer, const void* q_dev, cons
       !q_dev || !k_dev || !v_dev || !out_dev)
     return DMC_ERR_INVALID_ARG;
   return cuda_status(dmc::decode_launch(L, layer, c->Gv, c->decode_grid, c->decode_smem, q_dev,
+                                        k_dev, v_dev, out_dev, stream));
+}
+
+dmc_status dmc_decode_step_static_scratch(dmc_cache_t c, int32_t layer, const void* q_dev,
+                                          const void* k_dev, const void* v_dev, void* out_dev,
+                                          cudaStream_t stream) {
+  if (!c) return DMC_ERR_INVALID_ARG;
+  const Layout& L = c->lay;
+  if (layer < 0 || layer >= L.L) return DMC_ERR_INVALID_ARG;
+  if (!aligned16(q_dev) || !aligned16(k_dev) || !aligned16(v_dev) || !aligned16(out_dev) ||
+      !q_dev || !k_dev || !v_dev || !out_dev)
+    return DMC_ERR_INVALID_ARG;
+  int dev = -1;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return DMC_ERR_CUDA;
+  if (dev != c->device) return DMC_ERR_INVALID_ARG;
+  float* scratch = nullptr;
+  size_t floats = 0;
+  e = dmc::decode_static_partials(dev, &scratch, &floats);
+  if (e != cudaSuccess) return DMC_ERR_CUDA;
+  // two partial states of head_dim + 2 floats per block of the decode grid
+  if ((size_t)2 * c->decode_grid * (size_t)(L.D + 2) > floats) return DMC_ERR_INVALID_ARG;
+  Layout ls = L;
+  ls.partials = scratch;
+  return cuda_status(dmc::decode_launch(ls, layer, c->Gv, c->decode_grid, c->decode_smem, q_dev,
                                         k_dev, v_dev, out_dev, stream));
 }
 

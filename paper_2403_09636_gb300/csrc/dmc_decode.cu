@@ -26,6 +26,8 @@
 // when the launch is replayed from a CUDA graph.
 #include <math.h>
 
+#include <mutex>
+
 #include "dmc_internal.cuh"
 
 namespace dmc {
@@ -617,6 +619,33 @@ cudaError_t decode_launch(const Layout& L, int layer, int Gv, int grid, size_t s
   else
     return cudaErrorInvalidValue;
   return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------- static scratch
+// Scratch of dmc_decode_step_static_scratch: room for the split-K partial
+// softmax states of one launch (2 per block, head_dim <= 128, grid <= 1024
+// blocks), 1.04 MB. Every GPU that loads the library holds it until exit.
+constexpr size_t kStaticPartialFloats = (size_t)2 * kMaxDecodeBlocks * (128 + 2);
+static __device__ __align__(256) float g_decode_static_partials[kStaticPartialFloats];
+
+// Host code must not pass g_decode_static_partials itself to a kernel (on the
+// host it only names a stand-in). This looks up its device address once per
+// device, with that device current, and remembers it.
+cudaError_t decode_static_partials(int device, float** ptr, size_t* floats) {
+  constexpr int kMaxDevices = 64;
+  static std::mutex mu;
+  static float* addr[kMaxDevices] = {};
+  if (device < 0 || device >= kMaxDevices) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lock(mu);
+  if (addr[device] == nullptr) {
+    void* p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_decode_static_partials);
+    if (e != cudaSuccess) return e;
+    addr[device] = static_cast<float*>(p);
+  }
+  *ptr = addr[device];
+  *floats = kStaticPartialFloats;
+  return cudaSuccess;
 }
 
 }  // namespace dmc
