@@ -139,9 +139,9 @@ dmc_status dmc_decode_step(dmc_cache_t cache, int32_t layer, const void* q_dev,
  * implicit device synchronisation. Same arguments, semantics and results as
  * dmc_decode_step; it allocates nothing and calls no allocating routine.
  * The scratch is the split-K partial softmax states of one launch, kept in a
- * file-scope __device__ array of 1.04 MB (2 states of head_dim + 2 floats for
- * each of at most 1024 blocks) that every GPU loading the library holds until
- * the process exits; a cache whose decode grid would need more returns
+ * file-scope __device__ array of 4.26 MB (2 states of head_dim + 2 floats for
+ * each of at most 4096 worker warps) that every GPU loading the library holds
+ * until the process exits; a cache whose decode grid would need more returns
  * DMC_ERR_INVALID_ARG. Nothing in it needs to start at zero: each launch writes
  * every state before reading it. The first call on a device looks up the
  * array's device address on that device (which must be current and be the

@@ -9,15 +9,15 @@
 #include "dmc_internal.cuh"
 
 namespace dmc {
-cudaError_t decode_setup(const Layout& L, int Gv, int* grid, size_t* smem);
-cudaError_t decode_launch(const Layout& L, int layer, int Gv, int grid, size_t smem,
+cudaError_t decode_setup(const Layout& L, int Gv, DecodePlan* plan);
+cudaError_t decode_launch(const Layout& L, int layer, int Gv, const DecodePlan& plan, bool pdl,
                           const void* q, const void* k, const void* v, void* out,
                           cudaStream_t stream);
 cudaError_t prefill_launch(const Layout& L, int layer, int first_seq, int num_seqs, const void* q,
                            long long q_tok, long long q_head, const void* k, const void* v,
                            const int* cu, int total_tokens, int max_seqlen, cudaStream_t stream);
 cudaError_t decode_static_partials(int device, float** ptr, size_t* floats);
-constexpr int kMaxPartialBlocks = 1024;  // upper bound of the decode grid
+constexpr int kMaxPartialStates = 8192;  // two per decode worker warp (512 blocks x 8 warps)
 }  // namespace dmc
 
 using dmc::Layout;
@@ -27,8 +27,8 @@ struct dmc_cache {
   Layout lay;
   int device;
   int Gv;
-  int decode_grid;
-  size_t decode_smem;
+  dmc::DecodePlan plan;
+  int last_decode_layer;  // layer of the latest decode launch, -1 before any
   char* meta;  // lengths, ctl, counters, pool top, error: cleared by create / reset
   size_t meta_bytes;
 };
@@ -82,7 +82,7 @@ Offsets offsets(const dmc_cache_config* c) {
   o.pool_top = at; at = align_up(at + 8);
   o.error = at; at = align_up(at + 4);
   o.meta_end = at;
-  o.partials = at; at = align_up(at + (size_t)2 * dmc::kMaxPartialBlocks * (c->head_dim + 2) * 4);
+  o.partials = at; at = align_up(at + (size_t)dmc::kMaxPartialStates * (c->head_dim + 2) * 4);
   o.opens = at; at = align_up(at + (size_t)c->max_prefill_tokens * c->num_kv_heads);
   o.plan = at; at = align_up(at + (size_t)c->num_kv_heads * o.plan_stride * 4);
   o.total = at;
@@ -172,7 +172,7 @@ dmc_status dmc_cache_create(const dmc_cache_config* cfg, void* arena_dev, size_t
   L.pool_top = reinterpret_cast<unsigned long long*>(base + o.pool_top);
   L.error = reinterpret_cast<unsigned int*>(base + o.error);
   L.partials = reinterpret_cast<float*>(base + o.partials);
-  L.max_blocks = dmc::kMaxPartialBlocks;
+  L.max_blocks = dmc::kMaxPartialStates / 2;
   L.opens = reinterpret_cast<unsigned char*>(base + o.opens);
   L.plan = reinterpret_cast<int*>(base + o.plan);
   L.plan_stride = o.plan_stride;
@@ -180,8 +180,9 @@ dmc_status dmc_cache_create(const dmc_cache_config* cfg, void* arena_dev, size_t
   c->meta = base + o.meta;
   c->meta_bytes = o.meta_end - o.meta;
   c->Gv = L.G;  // one query head per unit list entry (G = 1 for MHA)
+  c->last_decode_layer = -1;
   cudaError_t e = cudaGetDevice(&c->device);
-  if (e == cudaSuccess) e = dmc::decode_setup(L, c->Gv, &c->decode_grid, &c->decode_smem);
+  if (e == cudaSuccess) e = dmc::decode_setup(L, c->Gv, &c->plan);
   if (e == cudaSuccess) e = cudaMemsetAsync(c->meta, 0, c->meta_bytes, stream);
   if (e != cudaSuccess) {
     delete c;
@@ -229,8 +230,12 @@ dmc_status dmc_decode_step(dmc_cache_t c, int32_t layer, const void* q_dev, cons
   if (!aligned16(q_dev) || !aligned16(k_dev) || !aligned16(v_dev) || !aligned16(out_dev) ||
       !q_dev || !k_dev || !v_dev || !out_dev)
     return DMC_ERR_INVALID_ARG;
-  return cuda_status(dmc::decode_launch(L, layer, c->Gv, c->decode_grid, c->decode_smem, q_dev,
-                                        k_dev, v_dev, out_dev, stream));
+  // The launch may overlap the previous kernel's tail unless that was a decode
+  // of this same layer (whose writes the prologue would read).
+  const bool pdl = layer != c->last_decode_layer;
+  c->last_decode_layer = layer;
+  return cuda_status(dmc::decode_launch(L, layer, c->Gv, c->plan, pdl, q_dev, k_dev, v_dev,
+                                        out_dev, stream));
 }
 
 dmc_status dmc_decode_step_static_scratch(dmc_cache_t c, int32_t layer, const void* q_dev,
@@ -251,11 +256,13 @@ dmc_status dmc_decode_step_static_scratch(dmc_cache_t c, int32_t layer, const vo
   e = dmc::decode_static_partials(dev, &scratch, &floats);
   if (e != cudaSuccess) return DMC_ERR_CUDA;
   // two partial states of head_dim + 2 floats per block of the decode grid
-  if ((size_t)2 * c->decode_grid * (size_t)(L.D + 2) > floats) return DMC_ERR_INVALID_ARG;
+  if ((size_t)c->plan.partial_states * (size_t)(L.D + 2) > floats) return DMC_ERR_INVALID_ARG;
   Layout ls = L;
   ls.partials = scratch;
-  return cuda_status(dmc::decode_launch(ls, layer, c->Gv, c->decode_grid, c->decode_smem, q_dev,
-                                        k_dev, v_dev, out_dev, stream));
+  const bool pdl = layer != c->last_decode_layer;
+  c->last_decode_layer = layer;
+  return cuda_status(dmc::decode_launch(ls, layer, c->Gv, c->plan, pdl, q_dev, k_dev, v_dev,
+                                        out_dev, stream));
 }
 
 dmc_status dmc_cache_lengths(dmc_cache_t c, int32_t layer, int32_t* out_dev, cudaStream_t stream) {

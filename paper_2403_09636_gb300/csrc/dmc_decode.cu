@@ -2,28 +2,38 @@
 // single-query softmax attention over each head's updated, variable-length,
 // paged cache (Eq. attn-softmax over the compressed slots, Sec. 3.1).
 //
-// Work split ("stream-K" over slot pages): every head h contributes
-// ceil(len_old(h) / 32) page units plus one "owner" unit that holds the token
-// being merged or appended. All units of a layer form one list; block b takes
-// the contiguous range [b*U/nb, (b+1)*U/nb), so every block streams the same
-// number of pages whatever the spread of head lengths. A head cut by a range
-// boundary is finished by whichever of its blocks arrives last (a counter, no
-// waiting): it merges the blocks' partial softmax states in a fixed order.
+// Work split: every head h contributes ceil(len_old(h) / 32) page units plus
+// one "owner" unit that carries the token being merged or appended. All units
+// of a layer form one list, split into equal contiguous ranges over every warp
+// of the grid ("stream-K" at warp granularity), so each warp streams the same
+// number of pages whatever the spread of head lengths. Warps are independent
+// workers: there is no barrier between them after the prologue.
 //
-// Inside a block one producer warp walks the range and issues TMA bulk copies
-// (cp.async.bulk) of each page's K rows and V rows into a ring of shared
-// memory stages; 8 consumer warps read them. A 32-slot page maps one slot row
-// onto each 8-lane group; a lane holds 16 bytes of the row per 128-byte chunk.
+// A warp streams its pages in "quads" of 4 slot rows, one row per 8-lane
+// group, 16 bytes per lane per 128-byte chunk of a row. Each lane copies its
+// own chunks of K and V with cp.async into a private ring of kRing quads in
+// shared memory and later reads back exactly the bytes it copied, so the ring
+// needs no synchronisation; kRing - 1 quads are in flight per warp. A head cut
+// by range boundaries is finished by whichever of its warps arrives last
+// (a counter, no waiting), which merges the partial softmax states in worker
+// order, so results are deterministic.
+//
 // The slot that Algorithm 1 changes (the merged last slot, or the new one) is
 // never read from the page: the owner unit computes it in registers from the
-// old row, z and the new k, v, stores it rounded to the cache dtype, and
-// scores that rounded value, so every block of the layer reads only slots this
-// launch does not write.
+// old row, z and the new k, v, stores it rounded to the cache dtype and scores
+// that rounded value, so no warp reads a slot the launch writes.
 //
-// Slot counts are double-buffered per layer: this launch reads buffer `parity`
-// and writes the other; the last block to finish flips the parity. That keeps
-// the unit list consistent while owners publish new lengths, and stays correct
-// when the launch is replayed from a CUDA graph.
+// Slot counts are double-buffered per layer: this launch reads buffer
+// `parity` and writes the other; the last block to finish flips the parity, so
+// the unit list stays consistent while owners publish new lengths, and a
+// replayed CUDA graph stays correct.
+//
+// Programmatic dependent launch: everything before griddep_wait() reads only
+// this layer's cache state (lengths, page table, pages), never q, k, v or
+// anything a preceding kernel of another layer writes, so it may overlap the
+// tail of the previous kernel on the stream. The host does not use the
+// attribute when the previous decode launch of the cache was for the same
+// layer.
 #include <math.h>
 
 #include <mutex>
@@ -32,23 +42,16 @@
 
 namespace dmc {
 
-constexpr int kConsumerWarps = 8;
-constexpr int kConsumers = kConsumerWarps * 32;
-constexpr int kDecodeThreads = kConsumers + 32;
-constexpr int kStages = 4;
-constexpr int kMaxDecodeBlocks = 1024;
+constexpr int kWarps = 8;  // independent workers per block
+constexpr int kDecodeThreads = kWarps * 32;
+constexpr int kRing = 6;        // quads per warp ring (kRing - 1 in flight)
+constexpr int kWindow = 64;     // page units per warp window (page id + rows to copy)
+constexpr int kHeadWindow = 32; // heads whose gates a warp holds in its lanes
+constexpr int kMaxDecodeBlocks = 512;
+constexpr int kMaxWorkers = kMaxDecodeBlocks * kWarps;
+static_assert(kMaxWorkers * 2 == 8192, "partials hold two states per worker");
 
 enum : int { kFlagAcc = 1, kFlagNaN = 2 };
-
-struct StageHdr {
-  int len_old;
-  int rows;      // fixed slot rows in this stage
-  int flags;     // kFlagAcc: owner unit merges into the last slot
-  int tgt_page;  // owner: page of the slot being written, -1 = allocate one
-  float omega;
-  int pad[11];
-};
-static_assert(sizeof(StageHdr) == 64, "header is 64 bytes");
 
 struct DecodeArgs {
   Layout lay;
@@ -63,35 +66,39 @@ struct DecodeArgs {
 template <typename T, int D>
 struct DecodeGeom {
   static constexpr int ROW = D * (int)sizeof(T);
-  static constexpr int NCH = ROW / 128;      // 16-byte chunks per lane of an 8-lane group
-  static constexpr int EPC = Chunk<T>::N;    // elements per chunk
-  static constexpr int EPL = NCH * EPC;      // elements of a row held by one lane
-  static constexpr int OFF_Q = 64;
-  static constexpr int OFF_KIN = OFF_Q + ROW;
-  static constexpr int OFF_VIN = OFF_KIN + ROW;
-  static constexpr int OFF_KOLD = OFF_VIN + ROW;
-  static constexpr int OFF_VOLD = OFF_KOLD + ROW;
-  static constexpr int OFF_Z = OFF_VOLD + ROW;
-  static constexpr int OFF_K = ((OFF_Z + kPage * 4) + 127) / 128 * 128;
-  static constexpr int OFF_V = OFF_K + kPage * ROW;
-  static constexpr int STAGE = OFF_V + kPage * ROW;
-  static constexpr int RING = kStages * STAGE;
-  static constexpr int OFF_BARS = RING;                       // full[S], empty[S]
-  static constexpr int OFF_RED = OFF_BARS + 2 * kStages * 8;  // [warps][D + 2] floats
-  static constexpr int OFF_MISC = OFF_RED + kConsumerWarps * (D + 2) * 4;  // 16 ints
-  static constexpr int OFF_U = OFF_MISC + 64;                 // [NVH + 1] ints
-  static size_t smem_bytes(int nvh) { return (size_t)OFF_U + (size_t)(nvh + 1) * 4; }
+  static constexpr int NCH = ROW / 128;    // 16-byte chunks per lane of an 8-lane group
+  static constexpr int EPC = Chunk<T>::N;  // elements per chunk
+  static constexpr int EPL = NCH * EPC;    // elements of a row held by one lane
+  // ring slot of one warp: [2 * NCH chunks][32 lanes][16 bytes], K chunks first
+  static constexpr int WSLOT = 2 * NCH * 32 * 16;
+  static constexpr int WRING = kRing * WSLOT;
+  static constexpr int WWIN = 2 * kWindow * 4;  // page ids, rows to copy
+  static constexpr int WARP_BYTES = WRING + WWIN;
+  static constexpr int MISC = 64;
+  static size_t smem_bytes(int nvh) {
+    return (size_t)kWarps * WARP_BYTES + MISC + (size_t)(nvh + 1) * 4;
+  }
 };
 
-// Block b owns units [range_start(b), range_start(b + 1)); when there are more
-// blocks than units some ranges are empty.
-__device__ __forceinline__ long long range_start(int b, long long U, int nb) {
-  return (long long)b * U / nb;
+// Worker w owns units [range_start(w), range_start(w + 1)); when there are
+// more workers than units some ranges are empty.
+__device__ __forceinline__ long long range_start(int w, long long U, int nw) {
+  return (long long)w * U / nw;
 }
 
-// Index of the (non-empty) block whose unit range holds unit u.
-__device__ __forceinline__ int block_of_unit(long long u, long long U, int nb) {
-  return (int)(((u + 1) * nb - 1) / U);
+// Index of the (non-empty) worker whose unit range holds unit u.
+__device__ __forceinline__ int worker_of_unit(long long u, long long U, int nw) {
+  return (int)(((u + 1) * nw - 1) / U);
+}
+
+// Largest v in [0, n) with U[v] <= u (U ascending, U[0] = 0).
+__device__ __forceinline__ int head_of_unit(const int* U, int n, int u) {
+  int lo = 0, hi = n - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (U[mid] <= u) lo = mid; else hi = mid - 1;
+  }
+  return lo;
 }
 
 // Exclusive prefix of units per virtual head into U[0..nvh], all threads.
@@ -125,10 +132,9 @@ __device__ void scan_units(int* U, int* wsum, const int* len_cur, int nvh, int G
   __syncthreads();
 }
 
-template <typename T, int D>
+template <int EPL>
 __device__ __forceinline__ void merge_state(float& m, float& l, float* acc, float m2, float l2,
                                             const float* acc2) {
-  constexpr int EPL = DecodeGeom<T, D>::EPL;
   const float mn = fmaxf(m, m2);
   const float c1 = (m == -INFINITY) ? 0.f : exp2f(m - mn);
   const float c2 = (m2 == -INFINITY) ? 0.f : exp2f(m2 - mn);
@@ -150,211 +156,171 @@ dmc_decode_kernel(const DecodeArgs a) {
   const int Gv = a.Gv;
   const int NVH = L.NH * Gv;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int nb = gridDim.x, bid = blockIdx.x;
   int* ctl = L.ctl + a.layer * 4;
   const int parity = *reinterpret_cast<volatile int*>(&ctl[0]);
   const int* len_cur = L.lengths + ((size_t)a.layer * 2 + parity) * L.NH;
   int* len_nxt = L.lengths + ((size_t)a.layer * 2 + (parity ^ 1)) * L.NH;
   int* ptab = L.page_table + (size_t)a.layer * L.NH * L.MPH;
 
-  const uint32_t bars = smem_u32(smem + G_::OFF_BARS);
-  auto full_bar = [&](int s) { return bars + 8u * s; };
-  auto empty_bar = [&](int s) { return bars + 8u * (kStages + s); };
-  float* red = reinterpret_cast<float*>(smem + G_::OFF_RED);
-  volatile int* misc = reinterpret_cast<volatile int*>(smem + G_::OFF_MISC);
-  int* U = reinterpret_cast<int*>(smem + G_::OFF_U);
+  unsigned char* ring = smem + (size_t)warp * G_::WARP_BYTES;
+  int* wpid = reinterpret_cast<int*>(ring + G_::WRING);
+  int* wrws = wpid + kWindow;
+  int* misc = reinterpret_cast<int*>(smem + (size_t)kWarps * G_::WARP_BYTES);
+  int* U = misc + G_::MISC / 4;
 
-  if (tid == 0) {
-    for (int s = 0; s < kStages; ++s) {
-      mbar_init(full_bar(s), 1);
-      mbar_init(empty_bar(s), kConsumerWarps);
-    }
-    fence_mbar_init();
-    misc[0] = 0;  // abort
-    misc[1] = 0;  // combine
-  }
-  scan_units(U, reinterpret_cast<int*>(smem + G_::OFF_MISC) + 4, len_cur, NVH, Gv);
-
+  // ---------------------------------------------------------------- prologue
+  scan_units(U, misc, len_cur, NVH, Gv);
   const long long Utot = U[NVH];
-  const int u0 = (int)((long long)bid * Utot / nb);
-  const int u1 = (int)((long long)(bid + 1) * Utot / nb);
+  const int NW = gridDim.x * kWarps;
+  const int wid = blockIdx.x * kWarps + warp;
+  const int u0 = (int)range_start(wid, Utot, NW);
+  const int u1 = (int)range_start(wid + 1, Utot, NW);
+  const int grp = lane >> 3, l8 = lane & 7;
+  const uint32_t ring_s = smem_u32(ring);
 
-  if (u0 < u1 && warp == kConsumerWarps) {
-    // ------------------------------------------------------------ producer warp
-    int vh = 0;
-    {  // largest vh with U[vh] <= u0
-      int lo = 0, hi = NVH - 1;
-      while (lo < hi) {
-        int mid = (lo + hi + 1) >> 1;
-        if (U[mid] <= u0) lo = mid; else hi = mid - 1;
+  // page window: page id and rows to copy of units [pb, pb + kWindow)
+  int pb = u0;
+  auto load_window = [&](int first) {
+    pb = first;
+    __syncwarp();
+    for (int i = lane; i < kWindow; i += 32) {
+      const int u = first + i;
+      int pid = 0, rws = 0;
+      if (u < u1) {
+        const int hv = head_of_unit(U, NVH, u);
+        const int j = u - U[hv];
+        if (j < U[hv + 1] - U[hv] - 1) {
+          const int bh = hv / Gv;
+          pid = ptab[(size_t)bh * L.MPH + j];
+          rws = min(kPage, len_cur[bh] - j * kPage);
+        }
       }
-      vh = lo;
+      wpid[i] = pid;
+      wrws[i] = rws;
     }
-    int bh = 0, len_old = 0, acc = 0, lfixed = 0, win_base = -1, win = 0;
-    float omega = 0.f;
-    bool nan_gate = false;
-    const int* pt_row = ptab;
-    int it = 0;
-    for (int u = u0; u < u1; ++u, ++it) {
-      while (U[vh + 1] <= u) ++vh;
-      const int hu0 = U[vh], nU = U[vh + 1] - hu0, j = u - hu0;
-      const bool first = (u == u0) || (j == 0);
-      if (first) {
-        bh = vh / Gv;
-        const int b = bh / L.Hkv, h = bh % L.Hkv;
-        len_old = len_cur[bh];
-        const float x = Elt<T>::to_f(reinterpret_cast<const T*>(a.k)[(size_t)bh * D]);
-        nan_gate = (x != x);
-        acc = (x >= 0.f && len_old > 0) ? 1 : 0;  // alpha = round(sigmoid(k[0])) = [k[0] >= 0]
-        lfixed = len_old - acc;                     // slots no unit of this launch writes
-        float q0 = 0.f;
-        if (lane < L.G)
-          q0 = Elt<T>::to_f(
-              reinterpret_cast<const T*>(a.q)[((size_t)b * L.Hq + (size_t)h * L.G + lane) * D]);
+    __syncwarp();
+  };
+
+  // issue cursor: the next quad to copy into the ring
+  int iu = u0, iq = 0, inq = -1, islot = 0;
+  auto issue_next = [&]() {
+    while (iu < u1) {
+      if (iu - pb >= kWindow) load_window(iu);
+      if (inq < 0) inq = (wrws[iu - pb] + 3) >> 2;
+      if (iq < inq) break;
+      ++iu;
+      iq = 0;
+      inq = -1;
+    }
+    if (iu < u1) {
+      const int row = iq * 4 + grp;
+      if (row < wrws[iu - pb]) {
+        const char* src = L.pages + (size_t)wpid[iu - pb] * L.page_bytes + (size_t)row * ROW + l8 * 16;
+        const uint32_t dst = ring_s + islot * G_::WSLOT + lane * 16;
 #pragma unroll
-        for (int off = 16; off > 0; off >>= 1) q0 += __shfl_xor_sync(0xffffffffu, q0, off);
-        omega = sigmoidf_(q0 / (float)L.G);  // omega = sigmoid(mean of the group's q[0])
-        pt_row = ptab + (size_t)bh * L.MPH;
-        win_base = -1;
-      }
-      const bool owner = (j == nU - 1);
-      const int rows = owner ? 0 : max(0, min(kPage, lfixed - j * kPage));
-      int page = 0;
-      if (rows > 0) {
-        const int wb = j >> 5;
-        if (wb != win_base) {
-          const int idx = wb * 32 + lane;
-          win = idx < L.MPH ? pt_row[idx] : 0;
-          win_base = wb;
-        }
-        page = __shfl_sync(0xffffffffu, win, j & 31);
-      }
-      int old_page = -1, tgt = -1;
-      if (owner) {
-        if (acc) {
-          old_page = pt_row[(len_old - 1) / kPage];
-          tgt = old_page;
-        } else if (len_old % kPage != 0) {
-          tgt = pt_row[len_old / kPage];
+        for (int c = 0; c < NCH; ++c) {
+          cp_async16(dst + c * 512, src + c * 128);
+          cp_async16(dst + (NCH + c) * 512, src + (size_t)kPage * ROW + c * 128);
         }
       }
-      const int st = it % kStages;
-      const uint32_t ph = (uint32_t)(it / kStages) & 1u;
-      if (lane == 0) {
-        bool ok = misc[0] == 0 && mbar_wait(empty_bar(st), ph ^ 1u, L.error);
-        if (!ok) {
-          misc[0] = 1;
-        } else {
-          unsigned char* stage = smem + (size_t)st * G_::STAGE;
-          StageHdr* hdr = reinterpret_cast<StageHdr*>(stage);
-          hdr->len_old = len_old;
-          hdr->rows = rows;
-          hdr->flags = (owner && acc ? kFlagAcc : 0) | (nan_gate ? kFlagNaN : 0);
-          hdr->tgt_page = tgt;
-          hdr->omega = omega;
-          uint32_t bytes = 0;
-          if (first) bytes += ROW;
-          if (rows) bytes += 2u * rows * ROW;
-          if (owner) bytes += 2u * ROW + (acc ? 2u * ROW + kPage * 4u : 0u);
-          const uint32_t fb = full_bar(st);
-          if (bytes == 0) {
-            mbar_arrive(fb);
-          } else {
-            mbar_arrive_expect_tx(fb, bytes);
-            const uint32_t sbase = smem_u32(stage);
-            if (first) {
-              const int b = bh / L.Hkv, h = bh % L.Hkv, g = vh % Gv;
-              bulk_g2s(sbase + G_::OFF_Q,
-                       a.q + ((size_t)b * L.Hq + (size_t)h * L.G + g) * ROW, ROW, fb);
-            }
-            if (rows) {
-              const char* pg = L.pages + (size_t)page * L.page_bytes;
-              bulk_g2s(sbase + G_::OFF_K, pg, rows * ROW, fb);
-              bulk_g2s(sbase + G_::OFF_V, pg + kPage * ROW, rows * ROW, fb);
-            }
-            if (owner) {
-              bulk_g2s(sbase + G_::OFF_KIN, a.k + (size_t)bh * ROW, ROW, fb);
-              bulk_g2s(sbase + G_::OFF_VIN, a.v + (size_t)bh * ROW, ROW, fb);
-              if (acc) {
-                const int r = (len_old - 1) % kPage;
-                const char* pg = L.pages + (size_t)old_page * L.page_bytes;
-                bulk_g2s(sbase + G_::OFF_KOLD, pg + (size_t)r * ROW, ROW, fb);
-                bulk_g2s(sbase + G_::OFF_VOLD, pg + (size_t)(kPage + r) * ROW, ROW, fb);
-                bulk_g2s(sbase + G_::OFF_Z, L.z + (size_t)old_page * kPage, kPage * 4, fb);
-              }
-            }
-          }
-        }
-      }
-      __syncwarp();
-      if (misc[0]) break;
+      ++iq;
     }
-    if (lane == 0 && misc[0]) {
-      // Aborted: let every copy already issued land before the block exits.
-      for (int k = max(0, it - kStages); k < it; ++k)
-        mbar_wait(full_bar(k % kStages), (uint32_t)(k / kStages) & 1u, L.error);
-    }
-  } else if (u0 < u1) {
-    // ------------------------------------------------------------ consumer warps
-    const int grp = warp * 4 + (lane >> 3);  // slot row of a page handled by this 8-lane group
-    const int l8 = lane & 7;
+    cp_async_commit();  // one group per call, possibly empty, on every lane
+    islot = (islot + 1 == kRing) ? 0 : islot + 1;
+  };
+
+  if (u0 < u1) {
+    load_window(u0);
+    for (int s = 0; s < kRing - 1; ++s) issue_next();
+  }
+
+  // q, k, v and the slots this launch writes are touched only after this point
+  griddep_wait();
+  griddep_launch_dependents();
+
+  if (u0 < u1) {
+    // lane i holds the gates of head hb + i
+    int hb = 0, t_len = 0, t_flags = 0;
+    float t_omega = 0.f;
+    auto load_heads = [&](int first) {
+      hb = first;
+      const int hv = first + lane;
+      t_len = 0;
+      t_flags = 0;
+      t_omega = 0.f;
+      if (hv < NVH && U[hv] < u1) {
+        const int bh = hv / Gv, b = bh / L.Hkv, h = bh % L.Hkv;
+        const int len = len_cur[bh];
+        const float x = Elt<T>::to_f(reinterpret_cast<const T*>(a.k)[(size_t)bh * D]);
+        float qs = 0.f;
+        for (int g = 0; g < L.G; ++g)
+          qs += Elt<T>::to_f(
+              reinterpret_cast<const T*>(a.q)[((size_t)b * L.Hq + (size_t)h * L.G + g) * D]);
+        t_len = len;
+        // alpha = round(sigmoid(k[0])) = [k[0] >= 0]; an empty head always appends
+        t_flags = ((x >= 0.f && len > 0) ? kFlagAcc : 0) | ((x != x) ? kFlagNaN : 0);
+        t_omega = sigmoidf_(qs / (float)L.G);  // omega = sigmoid(mean of the group's q[0])
+      }
+    };
+    int vh = head_of_unit(U, NVH, u0);
+    load_heads(vh);
+
     const float qscale = 1.4426950408889634f / sqrtf((float)D);  // log2(e) / sqrt(d_h)
-    float qf[EPL];
-    float m = -INFINITY, lsum = 0.f, acc[EPL];
+    float qf[EPL], acc[EPL];
+    float m = -INFINITY, lsum = 0.f;
 #pragma unroll
     for (int i = 0; i < EPL; ++i) { acc[i] = 0.f; qf[i] = 0.f; }
-    int vh = 0;
-    {
-      int lo = 0, hi = NVH - 1;
-      while (lo < hi) {
-        int mid = (lo + hi + 1) >> 1;
-        if (U[mid] <= u0) lo = mid; else hi = mid - 1;
-      }
-      vh = lo;
-    }
-    int it = 0;
-    for (int u = u0; u < u1; ++u, ++it) {
+    int len_old = 0, flags = 0, cslot = 0;
+    float omega = 0.f;
+
+    for (int u = u0; u < u1; ++u) {
       while (U[vh + 1] <= u) ++vh;
       const int hu0 = U[vh], nU = U[vh + 1] - hu0, j = u - hu0;
-      const bool first = (u == u0) || (j == 0);
       const bool owner = (j == nU - 1);
-      const bool seg_end = owner || (u == u1 - 1);
-      const int st = it % kStages;
-      const uint32_t ph = (uint32_t)(it / kStages) & 1u;
-      const unsigned char* stage = smem + (size_t)st * G_::STAGE;
-      bool have = misc[0] == 0 && mbar_wait(full_bar(st), ph, L.error);
-      if (!have) misc[0] = 1;
-      have = __shfl_sync(0xffffffffu, have ? 1 : 0, 0) != 0;
-      if (have) {
-        const StageHdr hdr = *reinterpret_cast<const StageHdr*>(stage);
-        if (first) {
+      const int bh = vh / Gv;
+      if (u == u0 || j == 0) {
+        if (vh - hb >= kHeadWindow) load_heads(vh);
+        const int src = vh - hb;
+        len_old = __shfl_sync(0xffffffffu, t_len, src);
+        flags = __shfl_sync(0xffffffffu, t_flags, src);
+        omega = __shfl_sync(0xffffffffu, t_omega, src);
+        const int b = bh / L.Hkv, h = bh % L.Hkv, g = vh % Gv;
+        const char* qrow = a.q + ((size_t)b * L.Hq + (size_t)h * L.G + g) * ROW;
 #pragma unroll
-          for (int c = 0; c < NCH; ++c) {
-            float f[EPC];
-            CK::unpack(*reinterpret_cast<const uint4*>(stage + G_::OFF_Q + c * 128 + l8 * 16), f);
+        for (int c = 0; c < NCH; ++c) {
+          float f[EPC];
+          CK::unpack(__ldg(reinterpret_cast<const uint4*>(qrow + c * 128 + l8 * 16)), f);
 #pragma unroll
-            for (int e = 0; e < EPC; ++e) qf[c * EPC + e] = f[e] * qscale;
-          }
-          if (l8 == 0) qf[0] = 0.f;  // q[0] is the importance gate, not a feature
+          for (int e = 0; e < EPC; ++e) qf[c * EPC + e] = f[e] * qscale;
         }
-        {
-          // Every lane scores a row (rows past hdr.rows hold stale data and
-          // are discarded) so the shuffles run with the whole warp.
-          const bool active = grp < hdr.rows;
-          const unsigned char* krow = stage + G_::OFF_K + grp * ROW;
-          const unsigned char* vrow = stage + G_::OFF_V + grp * ROW;
-          float s = 0.f;
+        if (l8 == 0) qf[0] = 0.f;  // q[0] is the importance gate, not a feature
+      }
+      const int accum = flags & kFlagAcc;
+      if (!owner) {
+        const int rows_copied = min(kPage, len_old - j * kPage);
+        const int rows = min(kPage, len_old - accum - j * kPage);  // the merged slot is excluded
+        const int nq = (rows_copied + 3) >> 2;
+        for (int qd = 0; qd < nq; ++qd) {
+          issue_next();
+          cp_async_wait<kRing - 1>();  // this lane's copies of quad qd have landed
+          const unsigned char* sl = ring + cslot * G_::WSLOT + lane * 16;
+          cslot = (cslot + 1 == kRing) ? 0 : cslot + 1;
+          float s0 = 0.f, s1 = 0.f;
 #pragma unroll
           for (int c = 0; c < NCH; ++c) {
             float f[EPC];
-            CK::unpack(*reinterpret_cast<const uint4*>(krow + c * 128 + l8 * 16), f);
+            CK::unpack(*reinterpret_cast<const uint4*>(sl + c * 512), f);
 #pragma unroll
-            for (int e = 0; e < EPC; ++e) s = fmaf(qf[c * EPC + e], f[e], s);
+            for (int e = 0; e < EPC; e += 2) {
+              s0 = fmaf(qf[c * EPC + e], f[e], s0);
+              s1 = fmaf(qf[c * EPC + e + 1], f[e + 1], s1);
+            }
           }
+          float s = s0 + s1;
           s += __shfl_xor_sync(0xffffffffu, s, 1);
           s += __shfl_xor_sync(0xffffffffu, s, 2);
           s += __shfl_xor_sync(0xffffffffu, s, 4);
-          if (active) {
+          if (qd * 4 + grp < rows) {
             const float mn = fmaxf(m, s);
             const float corr = exp2f(m - mn);
             const float p = exp2f(s - mn);
@@ -362,7 +328,7 @@ dmc_decode_kernel(const DecodeArgs a) {
 #pragma unroll
             for (int c = 0; c < NCH; ++c) {
               float f[EPC];
-              CK::unpack(*reinterpret_cast<const uint4*>(vrow + c * 128 + l8 * 16), f);
+              CK::unpack(*reinterpret_cast<const uint4*>(sl + (NCH + c) * 512), f);
 #pragma unroll
               for (int e = 0; e < EPC; ++e)
                 acc[c * EPC + e] = fmaf(acc[c * EPC + e], corr, p * f[e]);
@@ -370,97 +336,99 @@ dmc_decode_kernel(const DecodeArgs a) {
             m = mn;
           }
         }
-        if (owner && warp == 0 && lane < 8) {
-          // Algorithm 1 on the new token, in fp32, result rounded to the cache dtype.
-          const int bh = vh / Gv;
-          const bool accumulate = (hdr.flags & kFlagAcc) != 0;
-          const float w = hdr.omega;
-          const int len_old = hdr.len_old;
-          float zold = 0.f, znew = w;
-          if (accumulate) {
-            zold = reinterpret_cast<const float*>(stage + G_::OFF_Z)[(len_old - 1) % kPage];
-            znew = zold + w;
-          }
-          uint4 nk[NCH], nv[NCH];
-          float kr[EPL], vr[EPL];
-#pragma unroll
-          for (int c = 0; c < NCH; ++c) {
-            float kin[EPC], vin[EPC];
-            CK::unpack(*reinterpret_cast<const uint4*>(stage + G_::OFF_KIN + c * 128 + l8 * 16), kin);
-            CK::unpack(*reinterpret_cast<const uint4*>(stage + G_::OFF_VIN + c * 128 + l8 * 16), vin);
-            if (c == 0 && l8 == 0) kin[0] = 0.f;  // k[0] <- 0 (Algorithm 1)
-            float kn[EPC], vn[EPC];
-            if (accumulate) {
-              float ko[EPC], vo[EPC];
-              CK::unpack(*reinterpret_cast<const uint4*>(stage + G_::OFF_KOLD + c * 128 + l8 * 16), ko);
-              CK::unpack(*reinterpret_cast<const uint4*>(stage + G_::OFF_VOLD + c * 128 + l8 * 16), vo);
-#pragma unroll
-              for (int e = 0; e < EPC; ++e) {
-                kn[e] = (ko[e] * zold + kin[e] * w) / znew;
-                vn[e] = (vo[e] * zold + vin[e] * w) / znew;
-              }
-            } else {
-#pragma unroll
-              for (int e = 0; e < EPC; ++e) { kn[e] = kin[e]; vn[e] = vin[e]; }
-            }
-            nk[c] = CK::pack(kn);
-            nv[c] = CK::pack(vn);
-            CK::unpack(nk[c], kr + c * EPC);  // the stored (rounded) values
-            CK::unpack(nv[c], vr + c * EPC);
-          }
-          if (vh % Gv == 0) {  // one writer per KV head
-            const int slot = accumulate ? len_old - 1 : len_old;
-            bool ok = slot < L.max_slots;
-            if (!ok && l8 == 0) atomicOr(L.error, DMC_FAULT_SLOT_CAPACITY);
-            int page = hdr.tgt_page;
-            if (ok && page < 0) {
-              if (l8 == 0) {
-                const unsigned long long id = atomicAdd(L.pool_top, 1ull);
-                if (id >= (unsigned long long)L.num_pages) {
-                  atomicOr(L.error, DMC_FAULT_PAGES_EXHAUSTED);
-                  page = -1;
-                } else {
-                  page = (int)id;
-                  ptab[(size_t)bh * L.MPH + slot / kPage] = page;
-                }
-              }
-              page = __shfl_sync(0xffu, page, 0, 8);
-            }
-            ok = ok && page >= 0;
-            if (ok) {
-              char* dst = L.pages + (size_t)page * L.page_bytes + (size_t)(slot % kPage) * ROW;
-#pragma unroll
-              for (int c = 0; c < NCH; ++c) {
-                *reinterpret_cast<uint4*>(dst + c * 128 + l8 * 16) = nk[c];
-                *reinterpret_cast<uint4*>(dst + (size_t)kPage * ROW + c * 128 + l8 * 16) = nv[c];
-              }
-            }
-            if (l8 == 0) {
-              if (ok) L.z[(size_t)page * kPage + slot % kPage] = znew;
-              len_nxt[bh] = ok ? slot + 1 : len_old;
-              if (hdr.flags & kFlagNaN) atomicOr(L.error, DMC_FAULT_NAN_GATE);
-            }
-          }
-          float s = 0.f;
-#pragma unroll
-          for (int i = 0; i < EPL; ++i) s = fmaf(qf[i], kr[i], s);
-          s += __shfl_xor_sync(0xffu, s, 1);
-          s += __shfl_xor_sync(0xffu, s, 2);
-          s += __shfl_xor_sync(0xffu, s, 4);
-          const float mn = fmaxf(m, s);
-          const float corr = exp2f(m - mn);
-          const float p = exp2f(s - mn);
-          lsum = fmaf(lsum, corr, p);
-#pragma unroll
-          for (int i = 0; i < EPL; ++i) acc[i] = fmaf(acc[i], corr, p * vr[i]);
-          m = mn;
+      } else if (grp == 0) {
+        // Algorithm 1 on the new token, in fp32, result rounded to the cache dtype.
+        const int* pt_row = ptab + (size_t)bh * L.MPH;
+        int tgt = -1;
+        if (accum || len_old % kPage != 0) tgt = pt_row[(len_old - 1) / kPage];
+        float zold = 0.f, znew = omega;
+        const char* orow = nullptr;
+        if (accum) {
+          orow = L.pages + (size_t)tgt * L.page_bytes + (size_t)((len_old - 1) % kPage) * ROW;
+          zold = L.z[(size_t)tgt * kPage + (len_old - 1) % kPage];
+          znew = zold + omega;
         }
+        uint4 nk[NCH], nv[NCH];
+        float s = 0.f;
+#pragma unroll
+        for (int c = 0; c < NCH; ++c) {
+          float kin[EPC], vin[EPC];
+          CK::unpack(__ldg(reinterpret_cast<const uint4*>(a.k + (size_t)bh * ROW + c * 128 + l8 * 16)), kin);
+          CK::unpack(__ldg(reinterpret_cast<const uint4*>(a.v + (size_t)bh * ROW + c * 128 + l8 * 16)), vin);
+          if (c == 0 && l8 == 0) kin[0] = 0.f;  // k[0] <- 0 (Algorithm 1)
+          float kn[EPC], vn[EPC];
+          if (accum) {
+            float ko[EPC], vo[EPC];
+            CK::unpack(*reinterpret_cast<const uint4*>(orow + c * 128 + l8 * 16), ko);
+            CK::unpack(*reinterpret_cast<const uint4*>(orow + (size_t)kPage * ROW + c * 128 + l8 * 16), vo);
+#pragma unroll
+            for (int e = 0; e < EPC; ++e) {
+              kn[e] = (ko[e] * zold + kin[e] * omega) / znew;
+              vn[e] = (vo[e] * zold + vin[e] * omega) / znew;
+            }
+          } else {
+#pragma unroll
+            for (int e = 0; e < EPC; ++e) { kn[e] = kin[e]; vn[e] = vin[e]; }
+          }
+          nk[c] = CK::pack(kn);
+          nv[c] = CK::pack(vn);
+          float kr[EPC];
+          CK::unpack(nk[c], kr);  // score the stored (rounded) key
+#pragma unroll
+          for (int e = 0; e < EPC; ++e) s = fmaf(qf[c * EPC + e], kr[e], s);
+        }
+        if (vh % Gv == 0) {  // one writer per KV head
+          const int slot = accum ? len_old - 1 : len_old;
+          bool ok = slot < L.max_slots;
+          if (!ok && l8 == 0) atomicOr(L.error, DMC_FAULT_SLOT_CAPACITY);
+          int page = tgt;
+          if (ok && page < 0) {
+            if (l8 == 0) {
+              const unsigned long long id = atomicAdd(L.pool_top, 1ull);
+              if (id >= (unsigned long long)L.num_pages) {
+                atomicOr(L.error, DMC_FAULT_PAGES_EXHAUSTED);
+                page = -1;
+              } else {
+                page = (int)id;
+                ptab[(size_t)bh * L.MPH + slot / kPage] = page;
+              }
+            }
+            page = __shfl_sync(0xffu, page, 0, 8);
+          }
+          ok = ok && page >= 0;
+          if (ok) {
+            char* dst = L.pages + (size_t)page * L.page_bytes + (size_t)(slot % kPage) * ROW;
+#pragma unroll
+            for (int c = 0; c < NCH; ++c) {
+              *reinterpret_cast<uint4*>(dst + c * 128 + l8 * 16) = nk[c];
+              *reinterpret_cast<uint4*>(dst + (size_t)kPage * ROW + c * 128 + l8 * 16) = nv[c];
+            }
+          }
+          if (l8 == 0) {
+            if (ok) L.z[(size_t)page * kPage + slot % kPage] = znew;
+            len_nxt[bh] = ok ? slot + 1 : len_old;
+            if (flags & kFlagNaN) atomicOr(L.error, DMC_FAULT_NAN_GATE);
+          }
+        }
+        s += __shfl_xor_sync(0xffu, s, 1);
+        s += __shfl_xor_sync(0xffu, s, 2);
+        s += __shfl_xor_sync(0xffu, s, 4);
+        const float mn = fmaxf(m, s);
+        const float corr = exp2f(m - mn);
+        const float p = exp2f(s - mn);
+        lsum = fmaf(lsum, corr, p);
+#pragma unroll
+        for (int c = 0; c < NCH; ++c) {
+          float vr[EPC];
+          CK::unpack(nv[c], vr);
+#pragma unroll
+          for (int e = 0; e < EPC; ++e) acc[c * EPC + e] = fmaf(acc[c * EPC + e], corr, p * vr[e]);
+        }
+        m = mn;
       }
-      __syncwarp();
-      if (lane == 0) mbar_arrive(empty_bar(st));
 
-      if (seg_end) {
-        // ---- merge the 32 groups' softmax states, then emit or hand off
+      if (owner || u == u1 - 1) {
+        // ---- this warp's part of the head is done: merge its 4 groups
 #pragma unroll
         for (int off = 8; off < 32; off <<= 1) {
           const float m2 = __shfl_xor_sync(0xffffffffu, m, off);
@@ -468,82 +436,84 @@ dmc_decode_kernel(const DecodeArgs a) {
           float a2[EPL];
 #pragma unroll
           for (int i = 0; i < EPL; ++i) a2[i] = __shfl_xor_sync(0xffffffffu, acc[i], off);
-          merge_state<T, D>(m, lsum, acc, m2, l2, a2);
+          merge_state<EPL>(m, lsum, acc, m2, l2, a2);
         }
-        float* rw = red + warp * (D + 2);
-        if (lane == 0) { rw[0] = m; rw[1] = lsum; }
-        if (lane < 8) {
+        const int b = bh / L.Hkv, h = bh % L.Hkv, g = vh % Gv;
+        T* orow = reinterpret_cast<T*>(a.out) + ((size_t)b * L.Hq + (size_t)h * L.G + g) * D;
+        if (hu0 >= u0 && owner) {
+          // the whole head was in this warp
+          if (lane < 8) {
+            const float inv = 1.f / lsum;
 #pragma unroll
-          for (int c = 0; c < NCH; ++c)
+            for (int c = 0; c < NCH; ++c) {
+              float o[EPC];
 #pragma unroll
-            for (int e = 0; e < EPC; ++e)
-              rw[2 + (c * 128 + l8 * 16) / (int)sizeof(T) + e] = acc[c * EPC + e];
-        }
-        named_sync(1, kConsumers);
-        // block-level state for dimension tid (tid < D)
-        float M = -INFINITY;
-#pragma unroll
-        for (int w = 0; w < kConsumerWarps; ++w) M = fmaxf(M, red[w * (D + 2)]);
-        float Ls = 0.f, O = 0.f;
-#pragma unroll
-        for (int w = 0; w < kConsumerWarps; ++w) {
-          const float mw = red[w * (D + 2)];
-          const float cw = (mw == -INFINITY) ? 0.f : exp2f(mw - M);
-          Ls = fmaf(red[w * (D + 2) + 1], cw, Ls);
-          if (tid < D) O = fmaf(red[w * (D + 2) + 2 + tid], cw, O);
-        }
-        const int bh = vh / Gv, g = vh % Gv;
-        const int b = bh / L.Hkv, h = bh % L.Hkv;
-        const size_t orow = ((size_t)b * L.Hq + (size_t)h * L.G + g) * D;
-        const bool whole = (hu0 >= u0) && owner;
-        if (whole) {
-          if (tid < D) reinterpret_cast<T*>(a.out)[orow + tid] = Elt<T>::from_f(O / Ls);
+              for (int e = 0; e < EPC; ++e) o[e] = acc[c * EPC + e] * inv;
+              if constexpr (sizeof(T) == 2) {
+                *reinterpret_cast<uint4*>(orow + (c * 128 + l8 * 16) / 2) = CK::pack(o);
+              } else {
+                *reinterpret_cast<uint4*>(orow + (c * 128 + l8 * 16) / 4) = CK::pack(o);
+              }
+            }
+          }
         } else {
-          const int slot = 2 * bid + (hu0 <= u0 ? 0 : 1);
-          float* pp = L.partials + (size_t)slot * (D + 2);
-          if (tid == 0) { pp[0] = M; pp[1] = Ls; }
-          if (tid < D) pp[2 + tid] = O;
+          // publish this warp's partial state; the last contributor combines
+          const int ps = 2 * wid + (hu0 <= u0 ? 0 : 1);
+          float* pp = L.partials + (size_t)ps * (D + 2);
+          if (lane == 0) { pp[0] = m; pp[1] = lsum; }
+          if (lane < 8) {
+#pragma unroll
+            for (int c = 0; c < NCH; ++c)
+#pragma unroll
+              for (int e = 0; e < EPC; ++e)
+                pp[2 + (c * 128 + l8 * 16) / (int)sizeof(T) + e] = acc[c * EPC + e];
+          }
           __threadfence();
-          named_sync(1, kConsumers);
+          __syncwarp();
           const long long hend = U[vh + 1];
-          const int bf = block_of_unit(hu0, Utot, nb);
-          const int bl = block_of_unit(hend - 1, Utot, nb);
-          if (tid == 0) {
-            // contributors: the blocks of [bf, bl] with a non-empty unit range
+          const int wf = worker_of_unit(hu0, Utot, NW);
+          const int wl = worker_of_unit(hend - 1, Utot, NW);
+          int last = 0;
+          if (lane == 0) {
+            // contributors: the workers of [wf, wl] with a non-empty unit range
             int ncontrib = 0;
-            for (int cb = bf; cb <= bl; ++cb)
-              ncontrib += range_start(cb, Utot, nb) < range_start(cb + 1, Utot, nb);
+            for (int cw = wf; cw <= wl; ++cw)
+              ncontrib += range_start(cw, Utot, NW) < range_start(cw + 1, Utot, NW);
             int* cnt = L.counters + (size_t)a.layer * L.NH * L.G + vh;
             const int old = atomicAdd(cnt, 1);
-            const int last = (old == ncontrib - 1);
+            last = (old == ncontrib - 1);
             if (last) *cnt = 0;
-            misc[1] = last;
           }
-          named_sync(1, kConsumers);
-          if (misc[1]) {
+          last = __shfl_sync(0xffffffffu, last, 0);
+          if (last) {
             __threadfence();
+            constexpr int DPL = D / 32;  // output dims per lane
             float Mc = -INFINITY;
-            for (int cb = bf; cb <= bl; ++cb) {
-              const long long cstart = range_start(cb, Utot, nb);
-              if (cstart == range_start(cb + 1, Utot, nb)) continue;
-              const int cs = 2 * cb + (hu0 <= cstart ? 0 : 1);
+            for (int cw = wf; cw <= wl; ++cw) {
+              const long long cs0 = range_start(cw, Utot, NW);
+              if (cs0 == range_start(cw + 1, Utot, NW)) continue;
+              const int cs = 2 * cw + (hu0 <= cs0 ? 0 : 1);
               Mc = fmaxf(Mc, __ldcg(L.partials + (size_t)cs * (D + 2)));
             }
-            float Lc = 0.f, Oc = 0.f;
-            for (int cb = bf; cb <= bl; ++cb) {
-              const long long cstart = range_start(cb, Utot, nb);
-              if (cstart == range_start(cb + 1, Utot, nb)) continue;
-              const int cs = 2 * cb + (hu0 <= cstart ? 0 : 1);
+            float Lc = 0.f, Oc[DPL];
+#pragma unroll
+            for (int i = 0; i < DPL; ++i) Oc[i] = 0.f;
+            for (int cw = wf; cw <= wl; ++cw) {
+              const long long cs0 = range_start(cw, Utot, NW);
+              if (cs0 == range_start(cw + 1, Utot, NW)) continue;
+              const int cs = 2 * cw + (hu0 <= cs0 ? 0 : 1);
               const float* cp = L.partials + (size_t)cs * (D + 2);
               const float mc = __ldcg(cp);
-              const float cw = (mc == -INFINITY) ? 0.f : exp2f(mc - Mc);
-              Lc = fmaf(__ldcg(cp + 1), cw, Lc);
-              if (tid < D) Oc = fmaf(__ldcg(cp + 2 + tid), cw, Oc);
+              const float cwt = (mc == -INFINITY) ? 0.f : exp2f(mc - Mc);
+              Lc = fmaf(__ldcg(cp + 1), cwt, Lc);
+#pragma unroll
+              for (int i = 0; i < DPL; ++i) Oc[i] = fmaf(__ldcg(cp + 2 + lane * DPL + i), cwt, Oc[i]);
             }
-            if (tid < D) reinterpret_cast<T*>(a.out)[orow + tid] = Elt<T>::from_f(Oc / Lc);
+            const float inv = 1.f / Lc;
+#pragma unroll
+            for (int i = 0; i < DPL; ++i) orow[lane * DPL + i] = Elt<T>::from_f(Oc[i] * inv);
           }
         }
-        named_sync(1, kConsumers);  // `red` and misc[1] are reused by the next head
         m = -INFINITY;
         lsum = 0.f;
 #pragma unroll
@@ -551,12 +521,13 @@ dmc_decode_kernel(const DecodeArgs a) {
       }
     }
   }
+  cp_async_wait<0>();
 
   __syncthreads();
   if (tid == 0) {
     __threadfence();
     const int old = atomicAdd(&ctl[1], 1);
-    if (old == nb - 1) {  // last block of the launch: publish the new slot counts
+    if (old == (int)gridDim.x - 1) {  // last block of the launch: publish the new slot counts
       ctl[1] = 0;
       ctl[0] = parity ^ 1;
       __threadfence();
@@ -565,39 +536,60 @@ dmc_decode_kernel(const DecodeArgs a) {
 }
 
 template <typename T, int D>
-static cudaError_t setup_decode(int nvh, int* grid, size_t* smem) {
+static cudaError_t setup_decode(int nvh, DecodePlan* plan) {
   using G_ = DecodeGeom<T, D>;
-  *smem = G_::smem_bytes(nvh);
-  cudaError_t e = cudaFuncSetAttribute(dmc_decode_kernel<T, D>,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)*smem);
+  int dev = 0, sms = 0, optin = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
   if (e != cudaSuccess) return e;
-  int occ = 0, dev = 0, sms = 0;
-  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, dmc_decode_kernel<T, D>,
-                                                    kDecodeThreads, *smem);
+  plan->stages = kRing;
+  plan->smem = G_::smem_bytes(nvh);
+  if (plan->smem > (size_t)optin) return cudaErrorInvalidConfiguration;
+  e = cudaFuncSetAttribute(dmc_decode_kernel<T, D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           (int)plan->smem);
+  if (e != cudaSuccess) return e;
+  int occ = 0;
+  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, dmc_decode_kernel<T, D>, kDecodeThreads,
+                                                    plan->smem);
   if (e != cudaSuccess) return e;
   if (occ < 1) return cudaErrorInvalidConfiguration;
-  e = cudaGetDevice(&dev);
-  if (e != cudaSuccess) return e;
-  e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  if (e != cudaSuccess) return e;
-  *grid = min(sms * occ, kMaxDecodeBlocks);
+  plan->grid = min(sms * occ, kMaxDecodeBlocks);
   return cudaSuccess;
 }
 
-cudaError_t decode_setup(const Layout& L, int Gv, int* grid, size_t* smem) {
+cudaError_t decode_setup(const Layout& L, int Gv, DecodePlan* plan) {
   const int nvh = L.NH * Gv;
   cudaError_t e = cudaErrorInvalidValue;
-  if (L.esize == 4 && L.D == 64) e = setup_decode<float, 64>(nvh, grid, smem);
-  if (L.esize == 4 && L.D == 128) e = setup_decode<float, 128>(nvh, grid, smem);
-  if (L.esize == 2 && L.D == 64) e = setup_decode<__nv_bfloat16, 64>(nvh, grid, smem);
-  if (L.esize == 2 && L.D == 128) e = setup_decode<__nv_bfloat16, 128>(nvh, grid, smem);
-  // no more blocks than the most units a layer can have
+  if (L.esize == 4 && L.D == 64) e = setup_decode<float, 64>(nvh, plan);
+  if (L.esize == 4 && L.D == 128) e = setup_decode<float, 128>(nvh, plan);
+  if (L.esize == 2 && L.D == 64) e = setup_decode<__nv_bfloat16, 64>(nvh, plan);
+  if (L.esize == 2 && L.D == 128) e = setup_decode<__nv_bfloat16, 128>(nvh, plan);
+  // no more warps than the most units a layer can have
   const long long max_units = (long long)nvh * (L.MPH + 1);
-  if (e == cudaSuccess && max_units < *grid) *grid = (int)max_units;
+  const long long max_blocks = (max_units + kWarps - 1) / kWarps;
+  if (e == cudaSuccess && max_blocks < plan->grid) plan->grid = (int)max_blocks;
+  plan->partial_states = 2 * plan->grid * kWarps;
   return e;
 }
 
-cudaError_t decode_launch(const Layout& L, int layer, int Gv, int grid, size_t smem,
+template <typename T, int D>
+static cudaError_t launch_decode(const DecodeArgs& a, const DecodePlan& plan, bool pdl,
+                                 cudaStream_t stream) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(plan.grid);
+  cfg.blockDim = dim3(kDecodeThreads);
+  cfg.dynamicSmemBytes = plan.smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, dmc_decode_kernel<T, D>, a);
+}
+
+cudaError_t decode_launch(const Layout& L, int layer, int Gv, const DecodePlan& plan, bool pdl,
                           const void* q, const void* k, const void* v, void* out,
                           cudaStream_t stream) {
   DecodeArgs a;
@@ -608,24 +600,21 @@ cudaError_t decode_launch(const Layout& L, int layer, int Gv, int grid, size_t s
   a.k = static_cast<const char*>(k);
   a.v = static_cast<const char*>(v);
   a.out = static_cast<char*>(out);
-  if (L.esize == 4 && L.D == 64)
-    dmc_decode_kernel<float, 64><<<grid, kDecodeThreads, smem, stream>>>(a);
-  else if (L.esize == 4 && L.D == 128)
-    dmc_decode_kernel<float, 128><<<grid, kDecodeThreads, smem, stream>>>(a);
-  else if (L.esize == 2 && L.D == 64)
-    dmc_decode_kernel<__nv_bfloat16, 64><<<grid, kDecodeThreads, smem, stream>>>(a);
-  else if (L.esize == 2 && L.D == 128)
-    dmc_decode_kernel<__nv_bfloat16, 128><<<grid, kDecodeThreads, smem, stream>>>(a);
-  else
-    return cudaErrorInvalidValue;
+  cudaError_t e = cudaErrorInvalidValue;
+  if (L.esize == 4 && L.D == 64) e = launch_decode<float, 64>(a, plan, pdl, stream);
+  else if (L.esize == 4 && L.D == 128) e = launch_decode<float, 128>(a, plan, pdl, stream);
+  else if (L.esize == 2 && L.D == 64) e = launch_decode<__nv_bfloat16, 64>(a, plan, pdl, stream);
+  else if (L.esize == 2 && L.D == 128) e = launch_decode<__nv_bfloat16, 128>(a, plan, pdl, stream);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 
 // ---------------------------------------------------------------- static scratch
 // Scratch of dmc_decode_step_static_scratch: room for the split-K partial
-// softmax states of one launch (2 per block, head_dim <= 128, grid <= 1024
-// blocks), 1.04 MB. Every GPU that loads the library holds it until exit.
-constexpr size_t kStaticPartialFloats = (size_t)2 * kMaxDecodeBlocks * (128 + 2);
+// softmax states of one launch (2 per worker warp, head_dim <= 128, at most
+// 512 blocks of 8 warps), 4.26 MB. Every GPU that loads the library holds it
+// until exit.
+constexpr size_t kStaticPartialFloats = (size_t)2 * kMaxWorkers * (128 + 2);
 static __device__ __align__(256) float g_decode_static_partials[kStaticPartialFloats];
 
 // Host code must not pass g_decode_static_partials itself to a kernel (on the

@@ -40,6 +40,14 @@ struct Layout {
 
 __host__ __device__ inline int ceil_div(int a, int b) { return (a + b - 1) / b; }
 
+// Launch shape of the decode kernel for one cache, fixed at create time.
+struct DecodePlan {
+  int grid;            // blocks
+  int stages;          // shared-memory ring depth (quads per warp)
+  int partial_states;  // split-K partial states one launch may write
+  size_t smem;         // dynamic shared memory per block
+};
+
 // ---------------------------------------------------------------- dtype helpers
 template <typename T> struct Elt;
 template <> struct Elt<float> {
@@ -160,6 +168,26 @@ __device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t
           dst),
       "l"(src), "r"(bytes), "r"(bar)
       : "memory");
+}
+
+// cp.async (LDGSTS) of 16 bytes, L2 only, into this thread's shared memory.
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() {
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+// Waits until at most N of this thread's committed cp.async groups are pending.
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
+// Programmatic dependent launch: wait for the grid this one depends on (a
+// no-op when launched without the attribute), then let the next grid start.
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void griddep_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
 
 // Named barrier over the first `threads` threads of the block.
