@@ -102,13 +102,22 @@ __device__ __forceinline__ int head_of_unit(const int* U, int n, int u) {
 }
 
 // Exclusive prefix of units per virtual head into U[0..nvh], all threads.
-__device__ void scan_units(int* U, int* wsum, const int* len_cur, int nvh, int Gv) {
+// Reads both slot-count buffers together with the parity word, so the prefix
+// costs one round trip to memory.
+__device__ void scan_units(int* U, int* wsum, const int* ctl, const int* len_both, int nh,
+                           int nvh, int Gv) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int nthr = blockDim.x, nwarps = nthr >> 5;
   const int per = (nvh + nthr - 1) / nthr;
   const int i0 = min(tid * per, nvh), i1 = min(i0 + per, nvh);
+  const int parity = *reinterpret_cast<const volatile int*>(ctl);
   int local = 0;
-  for (int i = i0; i < i1; ++i) local += ceil_div(len_cur[i / Gv], kPage) + 1;
+  for (int i = i0; i < i1; ++i) {
+    const int l0 = len_both[i / Gv], l1 = len_both[nh + i / Gv];
+    const int units = ceil_div(parity ? l1 : l0, kPage) + 1;
+    U[i] = units;  // per-head count for now, prefixed below
+    local += units;
+  }
   int incl = local;
 #pragma unroll
   for (int off = 1; off < 32; off <<= 1) {
@@ -125,8 +134,9 @@ __device__ void scan_units(int* U, int* wsum, const int* len_cur, int nvh, int G
   __syncthreads();
   int run = wsum[warp] + incl - local;
   for (int i = i0; i < i1; ++i) {
+    const int units = U[i];
     U[i] = run;
-    run += ceil_div(len_cur[i / Gv], kPage) + 1;
+    run += units;
   }
   if (tid == 0) U[nvh] = wsum[nwarps];
   __syncthreads();
@@ -169,7 +179,7 @@ dmc_decode_kernel(const DecodeArgs a) {
   int* U = misc + G_::MISC / 4;
 
   // ---------------------------------------------------------------- prologue
-  scan_units(U, misc, len_cur, NVH, Gv);
+  scan_units(U, misc, ctl, L.lengths + (size_t)a.layer * 2 * L.NH, L.NH, NVH, Gv);
   const long long Utot = U[NVH];
   const int NW = gridDim.x * kWarps;
   const int wid = blockIdx.x * kWarps + warp;
@@ -177,6 +187,8 @@ dmc_decode_kernel(const DecodeArgs a) {
   const int u1 = (int)range_start(wid + 1, Utot, NW);
   const int grp = lane >> 3, l8 = lane & 7;
   const uint32_t ring_s = smem_u32(ring);
+
+  const int n = u1 - u0;
 
   // page window: page id and rows to copy of units [pb, pb + kWindow)
   int pb = u0;
@@ -201,18 +213,20 @@ dmc_decode_kernel(const DecodeArgs a) {
     __syncwarp();
   };
 
-  // issue cursor: the next quad to copy into the ring
-  int iu = u0, iq = 0, inq = -1, islot = 0;
+  // issue cursor: unit u0 + ik, quad iq of that unit
+  int ik = 0, iq = 0, inq = -1, islot = 0;
   auto issue_next = [&]() {
-    while (iu < u1) {
+    while (ik < n) {
+      const int iu = u0 + ik;
       if (iu - pb >= kWindow) load_window(iu);
       if (inq < 0) inq = (wrws[iu - pb] + 3) >> 2;
       if (iq < inq) break;
-      ++iu;
+      ++ik;
       iq = 0;
       inq = -1;
     }
-    if (iu < u1) {
+    if (ik < n) {
+      const int iu = u0 + ik;
       const int row = iq * 4 + grp;
       if (row < wrws[iu - pb]) {
         const char* src = L.pages + (size_t)wpid[iu - pb] * L.page_bytes + (size_t)row * ROW + l8 * 16;
@@ -264,6 +278,14 @@ dmc_decode_kernel(const DecodeArgs a) {
     };
     int vh = head_of_unit(U, NVH, u0);
     load_heads(vh);
+    // the query row of the next head, loaded ahead of its use
+    auto q_ptr = [&](int hv) {
+      const int bh = hv / Gv, b = bh / L.Hkv, h = bh % L.Hkv, g = hv % Gv;
+      return a.q + ((size_t)b * L.Hq + (size_t)h * L.G + g) * ROW + l8 * 16;
+    };
+    uint4 qraw[NCH];
+#pragma unroll
+    for (int c = 0; c < NCH; ++c) qraw[c] = __ldg(reinterpret_cast<const uint4*>(q_ptr(vh) + c * 128));
 
     const float qscale = 1.4426950408889634f / sqrtf((float)D);  // log2(e) / sqrt(d_h)
     float qf[EPL], acc[EPL];
@@ -273,27 +295,33 @@ dmc_decode_kernel(const DecodeArgs a) {
     int len_old = 0, flags = 0, cslot = 0;
     float omega = 0.f;
 
-    for (int u = u0; u < u1; ++u) {
+    for (int k = 0; k < n; ++k) {
+      const int u = u0 + k;
       while (U[vh + 1] <= u) ++vh;
-      const int hu0 = U[vh], nU = U[vh + 1] - hu0, j = u - hu0;
+      const int hu0 = U[vh], hend = U[vh + 1], nU = hend - hu0, j = u - hu0;
       const bool owner = (j == nU - 1);
       const int bh = vh / Gv;
-      if (u == u0 || j == 0) {
+      if (k == 0 || j == 0) {
         if (vh - hb >= kHeadWindow) load_heads(vh);
         const int src = vh - hb;
         len_old = __shfl_sync(0xffffffffu, t_len, src);
         flags = __shfl_sync(0xffffffffu, t_flags, src);
         omega = __shfl_sync(0xffffffffu, t_omega, src);
-        const int b = bh / L.Hkv, h = bh % L.Hkv, g = vh % Gv;
-        const char* qrow = a.q + ((size_t)b * L.Hq + (size_t)h * L.G + g) * ROW;
 #pragma unroll
         for (int c = 0; c < NCH; ++c) {
           float f[EPC];
-          CK::unpack(__ldg(reinterpret_cast<const uint4*>(qrow + c * 128 + l8 * 16)), f);
+          CK::unpack(qraw[c], f);
 #pragma unroll
           for (int e = 0; e < EPC; ++e) qf[c * EPC + e] = f[e] * qscale;
         }
         if (l8 == 0) qf[0] = 0.f;  // q[0] is the importance gate, not a feature
+        // prefetch the query of the head that follows in this range
+        const int next = hend < u1 ? vh + 1 : -1;
+        if (next >= 0) {
+#pragma unroll
+          for (int c = 0; c < NCH; ++c)
+            qraw[c] = __ldg(reinterpret_cast<const uint4*>(q_ptr(next) + c * 128));
+        }
       }
       const int accum = flags & kFlagAcc;
       if (!owner) {
@@ -427,7 +455,7 @@ dmc_decode_kernel(const DecodeArgs a) {
         m = mn;
       }
 
-      if (owner || u == u1 - 1) {
+      if (owner || k == n - 1) {
         // ---- this warp's part of the head is done: merge its 4 groups
 #pragma unroll
         for (int off = 8; off < 32; off <<= 1) {
@@ -440,7 +468,7 @@ dmc_decode_kernel(const DecodeArgs a) {
         }
         const int b = bh / L.Hkv, h = bh % L.Hkv, g = vh % Gv;
         T* orow = reinterpret_cast<T*>(a.out) + ((size_t)b * L.Hq + (size_t)h * L.G + g) * D;
-        if (hu0 >= u0 && owner) {
+        if (hu0 >= u0 && hend <= u1) {
           // the whole head was in this warp
           if (lane < 8) {
             const float inv = 1.f / lsum;
@@ -468,17 +496,21 @@ dmc_decode_kernel(const DecodeArgs a) {
               for (int e = 0; e < EPC; ++e)
                 pp[2 + (c * 128 + l8 * 16) / (int)sizeof(T) + e] = acc[c * EPC + e];
           }
-          __threadfence();
+          __threadfence();  // the partial is visible before the counter moves
           __syncwarp();
-          const long long hend = U[vh + 1];
           const int wf = worker_of_unit(hu0, Utot, NW);
           const int wl = worker_of_unit(hend - 1, Utot, NW);
+          // With at least one unit per worker every worker in [wf, wl] holds
+          // part of the head, and only wf can hold it as its last head.
+          const bool dense = Utot >= NW;
           int last = 0;
           if (lane == 0) {
-            // contributors: the workers of [wf, wl] with a non-empty unit range
-            int ncontrib = 0;
-            for (int cw = wf; cw <= wl; ++cw)
-              ncontrib += range_start(cw, Utot, NW) < range_start(cw + 1, Utot, NW);
+            int ncontrib = wl - wf + 1;
+            if (!dense) {
+              ncontrib = 0;
+              for (int cw = wf; cw <= wl; ++cw)
+                ncontrib += range_start(cw, Utot, NW) < range_start(cw + 1, Utot, NW);
+            }
             int* cnt = L.counters + (size_t)a.layer * L.NH * L.G + vh;
             const int old = atomicAdd(cnt, 1);
             last = (old == ncontrib - 1);
@@ -486,28 +518,56 @@ dmc_decode_kernel(const DecodeArgs a) {
           }
           last = __shfl_sync(0xffffffffu, last, 0);
           if (last) {
-            __threadfence();
+            __threadfence();  // every contributor's partial is visible to this lane
             constexpr int DPL = D / 32;  // output dims per lane
-            float Mc = -INFINITY;
-            for (int cw = wf; cw <= wl; ++cw) {
-              const long long cs0 = range_start(cw, Utot, NW);
-              if (cs0 == range_start(cw + 1, Utot, NW)) continue;
-              const int cs = 2 * cw + (hu0 <= cs0 ? 0 : 1);
-              Mc = fmaxf(Mc, __ldcg(L.partials + (size_t)cs * (D + 2)));
-            }
-            float Lc = 0.f, Oc[DPL];
+            float Oc[DPL];
 #pragma unroll
             for (int i = 0; i < DPL; ++i) Oc[i] = 0.f;
-            for (int cw = wf; cw <= wl; ++cw) {
-              const long long cs0 = range_start(cw, Utot, NW);
-              if (cs0 == range_start(cw + 1, Utot, NW)) continue;
-              const int cs = 2 * cw + (hu0 <= cs0 ? 0 : 1);
-              const float* cp = L.partials + (size_t)cs * (D + 2);
-              const float mc = __ldcg(cp);
-              const float cwt = (mc == -INFINITY) ? 0.f : exp2f(mc - Mc);
-              Lc = fmaf(__ldcg(cp + 1), cwt, Lc);
+            float Lc = 0.f;
+            if (dense && wl - wf < 32) {
+              // lane c reads contributor wf + c's (m, l); the dims are read in
+              // one pass of independent loads
+              const int nc = wl - wf + 1;
+              const int first_slot = (hu0 > range_start(wf, Utot, NW)) ? 1 : 0;
+              const int cs = 2 * (wf + lane) + (lane == 0 ? first_slot : 0);
+              float mc = -INFINITY, lc = 0.f;
+              if (lane < nc) {
+                mc = __ldcg(L.partials + (size_t)cs * (D + 2));
+                lc = __ldcg(L.partials + (size_t)cs * (D + 2) + 1);
+              }
+              float Mc = mc;
 #pragma unroll
-              for (int i = 0; i < DPL; ++i) Oc[i] = fmaf(__ldcg(cp + 2 + lane * DPL + i), cwt, Oc[i]);
+              for (int off = 16; off > 0; off >>= 1) Mc = fmaxf(Mc, __shfl_xor_sync(0xffffffffu, Mc, off));
+              const float wgt = (lane < nc && mc != -INFINITY) ? exp2f(mc - Mc) : 0.f;
+              Lc = lc * wgt;
+#pragma unroll
+              for (int off = 16; off > 0; off >>= 1) Lc += __shfl_xor_sync(0xffffffffu, Lc, off);
+              for (int c = 0; c < nc; ++c) {
+                const float w = __shfl_sync(0xffffffffu, wgt, c);
+                const int csc = __shfl_sync(0xffffffffu, cs, c);
+                const float* cp = L.partials + (size_t)csc * (D + 2) + 2 + lane * DPL;
+#pragma unroll
+                for (int i = 0; i < DPL; ++i) Oc[i] = fmaf(__ldcg(cp + i), w, Oc[i]);
+              }
+            } else {
+              float Mc = -INFINITY;
+              for (int cw = wf; cw <= wl; ++cw) {
+                const long long cs0 = range_start(cw, Utot, NW);
+                if (cs0 == range_start(cw + 1, Utot, NW)) continue;
+                const int cs = 2 * cw + (hu0 <= cs0 ? 0 : 1);
+                Mc = fmaxf(Mc, __ldcg(L.partials + (size_t)cs * (D + 2)));
+              }
+              for (int cw = wf; cw <= wl; ++cw) {
+                const long long cs0 = range_start(cw, Utot, NW);
+                if (cs0 == range_start(cw + 1, Utot, NW)) continue;
+                const int cs = 2 * cw + (hu0 <= cs0 ? 0 : 1);
+                const float* cp = L.partials + (size_t)cs * (D + 2);
+                const float mc = __ldcg(cp);
+                const float cwt = (mc == -INFINITY) ? 0.f : exp2f(mc - Mc);
+                Lc = fmaf(__ldcg(cp + 1), cwt, Lc);
+#pragma unroll
+                for (int i = 0; i < DPL; ++i) Oc[i] = fmaf(__ldcg(cp + 2 + lane * DPL + i), cwt, Oc[i]);
+              }
             }
             const float inv = 1.f / Lc;
 #pragma unroll
