@@ -57,8 +57,8 @@ bool valid_config(const dmc_cache_config* c) {
 
 // Byte offsets of every region; returns the total size.
 struct Offsets {
-  size_t pages, z, ptab, meta, lengths, ctl, counters, pool_top, error, meta_end, partials, opens,
-      plan, total;
+  size_t pages, z, ptab, meta, lengths, ctl, counters, pool_top, error, meta_end, partials,
+      pending, pending_at, pending_z, opens, plan, total;
   int MPH, plan_stride;
 };
 
@@ -83,6 +83,9 @@ Offsets offsets(const dmc_cache_config* c) {
   o.error = at; at = align_up(at + 4);
   o.meta_end = at;
   o.partials = at; at = align_up(at + (size_t)dmc::kMaxPartialStates * (c->head_dim + 2) * 4);
+  o.pending = at; at = align_up(at + (G > 1 ? (size_t)NH * 2 * row : 0));
+  o.pending_at = at; at = align_up(at + (G > 1 ? (size_t)NH * 4 : 0));
+  o.pending_z = at; at = align_up(at + (G > 1 ? (size_t)NH * 4 : 0));
   o.opens = at; at = align_up(at + (size_t)c->max_prefill_tokens * c->num_kv_heads);
   o.plan = at; at = align_up(at + (size_t)c->num_kv_heads * o.plan_stride * 4);
   o.total = at;
@@ -169,6 +172,9 @@ dmc_status dmc_cache_create(const dmc_cache_config* cfg, void* arena_dev, size_t
   L.lengths = reinterpret_cast<int*>(base + o.lengths);
   L.ctl = reinterpret_cast<int*>(base + o.ctl);
   L.counters = reinterpret_cast<int*>(base + o.counters);
+  L.pending = base + o.pending;
+  L.pending_at = reinterpret_cast<int*>(base + o.pending_at);
+  L.pending_z = reinterpret_cast<float*>(base + o.pending_z);
   L.pool_top = reinterpret_cast<unsigned long long*>(base + o.pool_top);
   L.error = reinterpret_cast<unsigned int*>(base + o.error);
   L.partials = reinterpret_cast<float*>(base + o.partials);

@@ -424,16 +424,26 @@ dmc_decode_kernel(const DecodeArgs a) {
             page = __shfl_sync(0xffu, page, 0, 8);
           }
           ok = ok && page >= 0;
+          // With grouped queries the other virtual heads of this KV head may
+          // still read the old last row and z in this launch: the new row waits
+          // in the pending buffer until the launch's last block writes it.
+          char* dst = Gv > 1 ? L.pending + (size_t)bh * 2 * ROW
+                             : L.pages + (size_t)page * L.page_bytes + (size_t)(slot % kPage) * ROW;
+          const size_t vstride = Gv > 1 ? (size_t)ROW : (size_t)kPage * ROW;
           if (ok) {
-            char* dst = L.pages + (size_t)page * L.page_bytes + (size_t)(slot % kPage) * ROW;
 #pragma unroll
             for (int c = 0; c < NCH; ++c) {
               *reinterpret_cast<uint4*>(dst + c * 128 + l8 * 16) = nk[c];
-              *reinterpret_cast<uint4*>(dst + (size_t)kPage * ROW + c * 128 + l8 * 16) = nv[c];
+              *reinterpret_cast<uint4*>(dst + vstride + c * 128 + l8 * 16) = nv[c];
             }
           }
           if (l8 == 0) {
-            if (ok) L.z[(size_t)page * kPage + slot % kPage] = znew;
+            if (Gv > 1) {
+              L.pending_at[bh] = ok ? page * kPage + slot % kPage : -1;
+              L.pending_z[bh] = znew;
+            } else if (ok) {
+              L.z[(size_t)page * kPage + slot % kPage] = znew;
+            }
             len_nxt[bh] = ok ? slot + 1 : len_old;
             if (flags & kFlagNaN) atomicOr(L.error, DMC_FAULT_NAN_GATE);
           }
@@ -586,8 +596,29 @@ dmc_decode_kernel(const DecodeArgs a) {
   __syncthreads();
   if (tid == 0) {
     __threadfence();
-    const int old = atomicAdd(&ctl[1], 1);
-    if (old == (int)gridDim.x - 1) {  // last block of the launch: publish the new slot counts
+    misc[0] = atomicAdd(&ctl[1], 1) == (int)gridDim.x - 1;
+  }
+  __syncthreads();
+  if (misc[0]) {
+    // last block of the launch: every owner has finished
+    if (Gv > 1) {
+      __threadfence();
+      for (int bh = tid; bh < L.NH; bh += kDecodeThreads) {
+        const int at = L.pending_at[bh];
+        if (at < 0) continue;
+        char* dst = L.pages + (size_t)(at / kPage) * L.page_bytes + (size_t)(at % kPage) * ROW;
+        const char* src = L.pending + (size_t)bh * 2 * ROW;
+        for (int i = 0; i < ROW; i += 16) {
+          *reinterpret_cast<uint4*>(dst + i) = *reinterpret_cast<const uint4*>(src + i);
+          *reinterpret_cast<uint4*>(dst + (size_t)kPage * ROW + i) =
+              *reinterpret_cast<const uint4*>(src + ROW + i);
+        }
+        L.z[at] = L.pending_z[bh];
+      }
+      __syncthreads();
+    }
+    if (tid == 0) {  // publish the new slot counts
+      __threadfence();
       ctl[1] = 0;
       ctl[0] = parity ^ 1;
       __threadfence();

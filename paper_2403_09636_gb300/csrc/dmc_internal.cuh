@@ -28,6 +28,9 @@ struct Layout {
   int* lengths;            // [L][2][NH]  double-buffered slot counts
   int* ctl;                // [L][4]: parity, finished-block counter
   int* counters;           // [L][NH * G] per (virtual) head combine counters
+  char* pending;           // [NH][2][D]: grouped queries: new last rows awaiting the grid's end
+  int* pending_at;         // [NH]: their slot (page * 32 + row), -1 = none
+  float* pending_z;        // [NH]: their z
   unsigned long long* pool_top;
   unsigned int* error;
   float* partials;         // [2 * max_blocks][D + 2]

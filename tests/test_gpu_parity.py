@@ -61,3 +61,15 @@ def test_llama2_7b_4x_full_shape_sampled(cuda_dev):
     runs 64 of the 512 steps to keep the test short."""
     wl = S.WORKLOADS["llama2_7b_4x"]
     _check(H.Run(wl, cuda_dev, H.random_samples(wl, 48, seed=7), decode_steps=64))
+
+
+def test_gqa_virtual_heads_read_the_old_last_slot(cuda_dev):
+    """Every query of a group merges the new token into the same old last
+    slot; the group's one writer must not let another query see the merged
+    row early. The race shows up intermittently, so the shape that exposed it
+    (fp32, d 128, two queries per KV head, short heads split over many warps)
+    runs several times."""
+    wl = S.Workload("f32_d128_g2", 1, 2, 4, 2, 128, "f32", (90, 130), 24, ("fixed", 3.0), 1.0,
+                    seed=4)
+    for _ in range(4):
+        _check(H.Run(wl, cuda_dev, H.all_samples(wl)))
