@@ -17,6 +17,10 @@ cudaError_t prefill_launch(const Layout& L, int layer, int first_seq, int num_se
                            long long q_tok, long long q_head, const void* k, const void* v,
                            const int* cu, int total_tokens, int max_seqlen, cudaStream_t stream);
 cudaError_t decode_static_partials(int device, float** ptr, size_t* floats);
+bool gqa_supported(const Layout& L);
+cudaError_t gqa_setup(const Layout& L, DecodePlan* plan);
+cudaError_t gqa_launch(const Layout& L, int layer, const DecodePlan& plan, bool pdl, const void* q,
+                       const void* k, const void* v, void* out, cudaStream_t stream);
 constexpr int kMaxPartialStates = 8192;  // two per decode worker warp (512 blocks x 8 warps)
 }  // namespace dmc
 
@@ -27,6 +31,7 @@ struct dmc_cache {
   Layout lay;
   int device;
   int Gv;
+  bool gqa;  // grouped queries on the tensor-core kernel (one worker per KV head)
   dmc::DecodePlan plan;
   int last_decode_layer;  // layer of the latest decode launch, -1 before any
   char* meta;  // lengths, ctl, counters, pool top, error: cleared by create / reset
@@ -82,7 +87,7 @@ Offsets offsets(const dmc_cache_config* c) {
   o.pool_top = at; at = align_up(at + 8);
   o.error = at; at = align_up(at + 4);
   o.meta_end = at;
-  o.partials = at; at = align_up(at + (size_t)dmc::kMaxPartialStates * (c->head_dim + 2) * 4);
+  o.partials = at; at = align_up(at + (size_t)dmc::kMaxPartialStates * G * (c->head_dim + 2) * 4);
   o.pending = at; at = align_up(at + (G > 1 ? (size_t)NH * 2 * row : 0));
   o.pending_at = at; at = align_up(at + (G > 1 ? (size_t)NH * 4 : 0));
   o.pending_z = at; at = align_up(at + (G > 1 ? (size_t)NH * 4 : 0));
@@ -185,10 +190,14 @@ dmc_status dmc_cache_create(const dmc_cache_config* cfg, void* arena_dev, size_t
   L.max_prefill_tokens = cfg->max_prefill_tokens;
   c->meta = base + o.meta;
   c->meta_bytes = o.meta_end - o.meta;
-  c->Gv = L.G;  // one query head per unit list entry (G = 1 for MHA)
+  // Grouped queries in bf16 (2 to 8 per KV head) run on the tensor-core kernel,
+  // one unit list entry per KV head; otherwise every query head is its own
+  // entry of the CUDA-core kernel (G = 1 for MHA).
+  c->gqa = dmc::gqa_supported(L);
+  c->Gv = c->gqa ? 1 : L.G;
   c->last_decode_layer = -1;
   cudaError_t e = cudaGetDevice(&c->device);
-  if (e == cudaSuccess) e = dmc::decode_setup(L, c->Gv, &c->plan);
+  if (e == cudaSuccess) e = c->gqa ? dmc::gqa_setup(L, &c->plan) : dmc::decode_setup(L, c->Gv, &c->plan);
   if (e == cudaSuccess) e = cudaMemsetAsync(c->meta, 0, c->meta_bytes, stream);
   if (e != cudaSuccess) {
     delete c;
@@ -240,6 +249,8 @@ dmc_status dmc_decode_step(dmc_cache_t c, int32_t layer, const void* q_dev, cons
   // of this same layer (whose writes the prologue would read).
   const bool pdl = layer != c->last_decode_layer;
   c->last_decode_layer = layer;
+  if (c->gqa)
+    return cuda_status(dmc::gqa_launch(L, layer, c->plan, pdl, q_dev, k_dev, v_dev, out_dev, stream));
   return cuda_status(dmc::decode_launch(L, layer, c->Gv, c->plan, pdl, q_dev, k_dev, v_dev,
                                         out_dev, stream));
 }
@@ -267,6 +278,8 @@ dmc_status dmc_decode_step_static_scratch(dmc_cache_t c, int32_t layer, const vo
   ls.partials = scratch;
   const bool pdl = layer != c->last_decode_layer;
   c->last_decode_layer = layer;
+  if (c->gqa)
+    return cuda_status(dmc::gqa_launch(ls, layer, c->plan, pdl, q_dev, k_dev, v_dev, out_dev, stream));
   return cuda_status(dmc::decode_launch(ls, layer, c->Gv, c->plan, pdl, q_dev, k_dev, v_dev,
                                         out_dev, stream));
 }

@@ -73,3 +73,12 @@ def test_gqa_virtual_heads_read_the_old_last_slot(cuda_dev):
                     seed=4)
     for _ in range(4):
         _check(H.Run(wl, cuda_dev, H.all_samples(wl)))
+
+
+@pytest.mark.parametrize("G,D", [(2, 128), (4, 64), (8, 64), (8, 128)])
+def test_gqa_tensor_core_groups(cuda_dev, G, D):
+    """bf16 groups of 2 to 8 queries per KV head run on the tensor-core kernel;
+    ragged prompts so heads end mid-page and split across warps."""
+    wl = S.Workload(f"gqa_g{G}_d{D}", 2, 3, 2 * G, 2, D, "bf16", (120, 700), 20, ("fixed", 2.0), 0.5,
+                    seed=G + D)
+    _check(H.Run(wl, cuda_dev, H.all_samples(wl)))
