@@ -36,8 +36,7 @@ sys.path.insert(0, ROOT)
 METRIC = "DMC decode tokens/s + HBM GB/s (% of ~8 TB/s) at 7B shape, 4x CR, 1 GB300"
 NOMINAL_HBM_GBS = 8000.0
 FALLBACK_HBM_GBS = 6800.0
-DECODE_SOURCES = ["paper_2403_09636_gb300/csrc/dmc_decode.cu",
-                  "paper_2403_09636_gb300/csrc/dmc_internal.cuh"]
+CSRC = "paper_2403_09636_gb300/csrc/"
 
 
 def log(*a):
@@ -72,24 +71,36 @@ def measured_peak():
         return FALLBACK_HBM_GBS, "fallback"
 
 
-def decode_source_sha():
+def decode_kernel(wl):
+    """(name, source files) of the decode kernel a cache of this shape runs:
+    bf16 groups of 2 to 8 queries per KV head take the tensor-core kernel."""
+    if wl.esize == 2 and 2 <= wl.group <= 8:
+        return (f"dmc_decode_gqa_kernel<{wl.head_dim}>",
+                [CSRC + "dmc_decode_gqa.cu", CSRC + "dmc_internal.cuh", CSRC + "dmc_split.cuh"])
+    return (f"dmc_decode_kernel<{wl.dtype},{wl.head_dim}>",
+            [CSRC + "dmc_decode.cu", CSRC + "dmc_internal.cuh", CSRC + "dmc_split.cuh"])
+
+
+def decode_source_sha(sources):
     h = hashlib.sha256()
-    for f in DECODE_SOURCES:
+    for f in sources:
         h.update(open(os.path.join(ROOT, f), "rb").read())
     return h.hexdigest()[:16]
 
 
-def committed_traffic(workload):
-    """dram bytes per decode launch from the committed ncu summary, if it was
-    taken on the current decode kernel source; else None."""
+def committed_traffic(workload, sources, per_launch_bytes):
+    """DRAM bytes per decode launch from the committed ncu capture, if it was
+    taken on the current decode kernel source, else None. The capture runs a
+    smaller case of the same per-layer shape; its DRAM bytes scale to this
+    run's launch by the algorithmic bytes (slots streamed) of each."""
     p = os.path.join(ROOT, "profiles", f"dmc_decode_{workload}.traffic.json")
     try:
         j = json.load(open(p))
     except Exception:
         return None
-    if j.get("source_sha") != decode_source_sha():
+    if j.get("source_sha") != decode_source_sha(sources):
         return None
-    return j.get("dram_bytes_per_launch")
+    return per_launch_bytes * j["captured_dram_bytes"] / j["captured_algorithmic_bytes"]
 
 
 class ClockSampler:
@@ -346,7 +357,8 @@ def run_ours(args, rank, world, dist):
     per_launch_bytes = dec_bytes / n_dec_launch
     achieved = per_launch_bytes / avg_launch_s / 1e9
     peak, peak_kind = measured_peak()
-    traffic = committed_traffic(args.workload)
+    kname, ksources = decode_kernel(wl)
+    traffic = committed_traffic(args.workload, ksources, per_launch_bytes)
     res = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": K,
         "warmup": args.warmup, "ms_per_step": total_ms / K, "higher_is_better": True,
@@ -364,8 +376,7 @@ def run_ours(args, rank, world, dist):
         "decode_frac_of_8tbs": achieved / NOMINAL_HBM_GBS,
         "prefill_hbm_gbs": K * pf_bytes / (pf_ms / 1e3) / 1e9,
         "slots_per_head_mean": slots_read / (n_dec_launch * n_heads),
-        "roofline": {"kernel": "dmc_decode_kernel<bf16,128>" if esize == 2 and D == 128 else
-                     "dmc_decode_kernel", "bound": "hbm", "achieved": achieved, "peak": peak,
+        "roofline": {"kernel": kname, "bound": "hbm", "achieved": achieved, "peak": peak,
                      "peak_kind": f"{peak_kind} copy bandwidth", "unit": "GB/s",
                      "frac": achieved / peak, "traffic": traffic,
                      "algorithmic_bytes_per_launch": per_launch_bytes,
