@@ -21,7 +21,11 @@ bool gqa_supported(const Layout& L);
 cudaError_t gqa_setup(const Layout& L, DecodePlan* plan);
 cudaError_t gqa_launch(const Layout& L, int layer, const DecodePlan& plan, bool pdl, const void* q,
                        const void* k, const void* v, void* out, cudaStream_t stream);
-constexpr int kMaxPartialStates = 8192;  // two per decode worker warp (512 blocks x 8 warps)
+// Split-K partial states a cache's arena holds: two per worker warp of the
+// decode grid (at most 512 blocks x 8 warps), times the group size for the
+// tensor-core kernel, which keeps one per query.
+constexpr int kMaxWorkerStates = 8192;
+inline size_t partial_states_cap(int G) { return (size_t)kMaxWorkerStates * G; }
 }  // namespace dmc
 
 using dmc::Layout;
@@ -33,7 +37,7 @@ struct dmc_cache {
   int Gv;
   bool gqa;  // grouped queries on the tensor-core kernel (one worker per KV head)
   dmc::DecodePlan plan;
-  int last_decode_layer;  // layer of the latest decode launch, -1 before any
+  int last_decode_layer;  // layer of the latest kernel if it was a decode, else -1
   char* meta;  // lengths, ctl, counters, pool top, error: cleared by create / reset
   size_t meta_bytes;
 };
@@ -87,7 +91,7 @@ Offsets offsets(const dmc_cache_config* c) {
   o.pool_top = at; at = align_up(at + 8);
   o.error = at; at = align_up(at + 4);
   o.meta_end = at;
-  o.partials = at; at = align_up(at + (size_t)dmc::kMaxPartialStates * G * (c->head_dim + 2) * 4);
+  o.partials = at; at = align_up(at + dmc::partial_states_cap(G) * (c->head_dim + 4) * 4);
   o.pending = at; at = align_up(at + (G > 1 ? (size_t)NH * 2 * row : 0));
   o.pending_at = at; at = align_up(at + (G > 1 ? (size_t)NH * 4 : 0));
   o.pending_z = at; at = align_up(at + (G > 1 ? (size_t)NH * 4 : 0));
@@ -183,7 +187,7 @@ dmc_status dmc_cache_create(const dmc_cache_config* cfg, void* arena_dev, size_t
   L.pool_top = reinterpret_cast<unsigned long long*>(base + o.pool_top);
   L.error = reinterpret_cast<unsigned int*>(base + o.error);
   L.partials = reinterpret_cast<float*>(base + o.partials);
-  L.max_blocks = dmc::kMaxPartialStates / 2;
+  L.partial_cap = (int)dmc::partial_states_cap(L.G);
   L.opens = reinterpret_cast<unsigned char*>(base + o.opens);
   L.plan = reinterpret_cast<int*>(base + o.plan);
   L.plan_stride = o.plan_stride;
@@ -207,6 +211,16 @@ dmc_status dmc_cache_create(const dmc_cache_config* cfg, void* arena_dev, size_t
   return DMC_OK;
 }
 
+// A decode launch may overlap the tail of the kernel before it on the stream
+// (programmatic dependent launch) only if that kernel was this cache's decode
+// of another layer: its prologue reads the layer's slot counts, page table and
+// pages, which this cache's prefill and decode of the same layer write.
+bool use_pdl(dmc_cache* c, int layer) {
+  const bool pdl = c->last_decode_layer >= 0 && c->last_decode_layer != layer;
+  c->last_decode_layer = layer;
+  return pdl;
+}
+
 dmc_status dmc_cache_destroy(dmc_cache_t cache) {
   delete cache;
   return DMC_OK;
@@ -214,6 +228,7 @@ dmc_status dmc_cache_destroy(dmc_cache_t cache) {
 
 dmc_status dmc_cache_reset(dmc_cache_t c, cudaStream_t stream) {
   if (!c) return DMC_ERR_INVALID_ARG;
+  c->last_decode_layer = -1;
   return cuda_status(cudaMemsetAsync(c->meta, 0, c->meta_bytes, stream));
 }
 
@@ -232,6 +247,7 @@ dmc_status dmc_prefill_compress(dmc_cache_t c, int32_t layer, int32_t first_seq,
   if (!q_dev || !k_dev || !v_dev || !cu_seqlens_dev || !aligned16(k_dev) || !aligned16(v_dev))
     return DMC_ERR_INVALID_ARG;
   if (q_token_stride < 0 || q_head_stride < 0) return DMC_ERR_INVALID_ARG;
+  c->last_decode_layer = -1;
   return cuda_status(dmc::prefill_launch(L, layer, first_seq, num_seqs, q_dev, q_token_stride,
                                          q_head_stride, k_dev, v_dev, cu_seqlens_dev, total_tokens,
                                          max_seqlen, stream));
@@ -245,10 +261,7 @@ dmc_status dmc_decode_step(dmc_cache_t c, int32_t layer, const void* q_dev, cons
   if (!aligned16(q_dev) || !aligned16(k_dev) || !aligned16(v_dev) || !aligned16(out_dev) ||
       !q_dev || !k_dev || !v_dev || !out_dev)
     return DMC_ERR_INVALID_ARG;
-  // The launch may overlap the previous kernel's tail unless that was a decode
-  // of this same layer (whose writes the prologue would read).
-  const bool pdl = layer != c->last_decode_layer;
-  c->last_decode_layer = layer;
+  const bool pdl = use_pdl(c, layer);
   if (c->gqa)
     return cuda_status(dmc::gqa_launch(L, layer, c->plan, pdl, q_dev, k_dev, v_dev, out_dev, stream));
   return cuda_status(dmc::decode_launch(L, layer, c->Gv, c->plan, pdl, q_dev, k_dev, v_dev,
@@ -272,12 +285,14 @@ dmc_status dmc_decode_step_static_scratch(dmc_cache_t c, int32_t layer, const vo
   size_t floats = 0;
   e = dmc::decode_static_partials(dev, &scratch, &floats);
   if (e != cudaSuccess) return DMC_ERR_CUDA;
-  // two partial states of head_dim + 2 floats per block of the decode grid
-  if ((size_t)c->plan.partial_states * (size_t)(L.D + 2) > floats) return DMC_ERR_INVALID_ARG;
+  // the launch's partial states (head_dim + 4 floats each for the CUDA-core
+  // kernel, head_dim + 2 for the tensor-core kernel) must fit
+  const size_t fit = floats / (size_t)(L.D + (c->gqa ? 2 : 4));
+  if ((size_t)c->plan.partial_states > fit) return DMC_ERR_INVALID_ARG;
   Layout ls = L;
   ls.partials = scratch;
-  const bool pdl = layer != c->last_decode_layer;
-  c->last_decode_layer = layer;
+  ls.partial_cap = (int)fit;
+  const bool pdl = use_pdl(c, layer);
   if (c->gqa)
     return cuda_status(dmc::gqa_launch(ls, layer, c->plan, pdl, q_dev, k_dev, v_dev, out_dev, stream));
   return cuda_status(dmc::decode_launch(ls, layer, c->Gv, c->plan, pdl, q_dev, k_dev, v_dev,

@@ -93,12 +93,106 @@ __device__ __forceinline__ void merge_state(float& m, float& l, float* acc, floa
   m = mn;
 }
 
+// Floats per split-K partial state: m, l, two pad words, then the D
+// accumulator floats, so the accumulator is 16-byte aligned.
+template <int D>
+constexpr int kPartialStride = D + 4;
+
+// The last contributor of a split head merges the nc partial states of workers
+// wf..wf+nc-1 in worker order and writes the head's output row. Lane
+// (cg = lane / 8, dg = lane % 8) sums contributors cg, cg + 4, ... over dims
+// [dg * D / 8, (dg + 1) * D / 8), eight contributors' loads in flight per
+// batch; the four contributor groups are then added with shuffles.
+template <typename T, int D>
+__device__ __noinline__ void combine_partials(const float* partials, int wf, int first_off,
+                                                 int nc, int lane, T* orow) {
+  constexpr int PS = kPartialStride<D>;
+  constexpr int V4 = D / 32;  // float4 per lane per contributor
+  const int cg = lane >> 3, dg = lane & 7;
+  auto slot = [&](int i) { return 2 * (wf + i) + (i == 0 ? first_off : 0); };
+  float2 ml0 = make_float2(-INFINITY, 0.f);
+  if (lane < nc) ml0 = __ldcg(reinterpret_cast<const float2*>(partials + (size_t)slot(lane) * PS));
+  float Mc = ml0.x;
+  for (int i = lane + 32; i < nc; i += 32) Mc = fmaxf(Mc, __ldcg(partials + (size_t)slot(i) * PS));
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) Mc = fmaxf(Mc, __shfl_xor_sync(0xffffffffu, Mc, off));
+  float Lc = 0.f;
+  float4 o[V4];
+#pragma unroll
+  for (int k = 0; k < V4; ++k) o[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+  for (int i0 = 0; i0 < nc; i0 += 32) {
+    const int i = i0 + lane;
+    float2 ml = ml0;
+    if (i0 > 0)
+      ml = i < nc ? __ldcg(reinterpret_cast<const float2*>(partials + (size_t)slot(i) * PS))
+                  : make_float2(-INFINITY, 0.f);
+    const float w = (i < nc && ml.x != -INFINITY) ? exp2f(ml.x - Mc) : 0.f;
+    Lc = fmaf(ml.y, w, Lc);
+    const int n32 = min(32, nc - i0);
+    for (int c0 = 0; c0 < n32; c0 += 8) {
+      float4 v[2][V4];
+      float wv[2];
+#pragma unroll
+      for (int r = 0; r < 2; ++r) {
+        const int c = c0 + 4 * r + cg;  // < 32
+        wv[r] = __shfl_sync(0xffffffffu, w, c);
+        if (c < n32) {
+          const float4* p = reinterpret_cast<const float4*>(partials + (size_t)slot(i0 + c) * PS + 4) + dg * V4;
+#pragma unroll
+          for (int k = 0; k < V4; ++k) v[r][k] = __ldcg(p + k);
+        } else {
+          wv[r] = 0.f;
+#pragma unroll
+          for (int k = 0; k < V4; ++k) v[r][k] = make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+      }
+#pragma unroll
+      for (int r = 0; r < 2; ++r)
+#pragma unroll
+        for (int k = 0; k < V4; ++k) {
+          o[k].x = fmaf(v[r][k].x, wv[r], o[k].x);
+          o[k].y = fmaf(v[r][k].y, wv[r], o[k].y);
+          o[k].z = fmaf(v[r][k].z, wv[r], o[k].z);
+          o[k].w = fmaf(v[r][k].w, wv[r], o[k].w);
+        }
+    }
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) Lc += __shfl_xor_sync(0xffffffffu, Lc, off);
+#pragma unroll
+  for (int k = 0; k < V4; ++k)
+#pragma unroll
+    for (int off = 8; off < 32; off <<= 1) {
+      o[k].x += __shfl_xor_sync(0xffffffffu, o[k].x, off);
+      o[k].y += __shfl_xor_sync(0xffffffffu, o[k].y, off);
+      o[k].z += __shfl_xor_sync(0xffffffffu, o[k].z, off);
+      o[k].w += __shfl_xor_sync(0xffffffffu, o[k].w, off);
+    }
+  if (cg == 0) {
+    const float inv = 1.f / Lc;
+    float f[4 * V4];
+#pragma unroll
+    for (int k = 0; k < V4; ++k) {
+      f[4 * k] = o[k].x * inv;
+      f[4 * k + 1] = o[k].y * inv;
+      f[4 * k + 2] = o[k].z * inv;
+      f[4 * k + 3] = o[k].w * inv;
+    }
+    constexpr int EPC = Chunk<T>::N;
+    char* dst = reinterpret_cast<char*>(orow) + (size_t)dg * (D / 8) * sizeof(T);
+#pragma unroll
+    for (int c = 0; c < 4 * V4 / EPC; ++c)
+      *reinterpret_cast<uint4*>(dst + c * 16) = Chunk<T>::pack(f + c * EPC);
+  }
+}
+
 template <typename T, int D>
 __global__ void __launch_bounds__(kDecodeThreads, 2)
 dmc_decode_kernel(const DecodeArgs a) {
   using G_ = DecodeGeom<T, D>;
   using CK = Chunk<T>;
   constexpr int ROW = G_::ROW, NCH = G_::NCH, EPC = G_::EPC, EPL = G_::EPL;
+  constexpr int PSTRIDE = kPartialStride<D>;
   extern __shared__ __align__(128) unsigned char smem[];
 
   const Layout& L = a.lay;
@@ -436,21 +530,24 @@ dmc_decode_kernel(const DecodeArgs a) {
         } else {
           // publish this warp's partial state; the last contributor combines
           const int ps = 2 * wid + (hu0 <= u0 ? 0 : 1);
-          float* pp = L.partials + (size_t)ps * (D + 2);
-          if (lane == 0) { pp[0] = m; pp[1] = lsum; }
-          if (lane < 8) {
+          float* pp = L.partials + (size_t)ps * PSTRIDE;
+          if (lane == 0) *reinterpret_cast<float2*>(pp) = make_float2(m, lsum);
+          // lanes of group g write float4 number g, g + 4, ... of their dims
 #pragma unroll
-            for (int c = 0; c < NCH; ++c)
-#pragma unroll
-              for (int e = 0; e < EPC; ++e)
-                pp[2 + (c * 128 + l8 * 16) / (int)sizeof(T) + e] = acc[c * EPC + e];
+          for (int v = 0; v < EPL / 4; ++v) {
+            if ((v & 3) == grp) {
+              const int c = v / (EPC / 4), e = (v % (EPC / 4)) * 4;
+              *reinterpret_cast<float4*>(pp + 4 + (c * 128 + l8 * 16) / (int)sizeof(T) + e) =
+                  make_float4(acc[c * EPC + e], acc[c * EPC + e + 1], acc[c * EPC + e + 2],
+                              acc[c * EPC + e + 3]);
+            }
           }
           __threadfence();  // the partial is visible before the counter moves
           __syncwarp();
           const int wf = worker_of_unit(hu0, Utot, NW);
           const int wl = worker_of_unit(hend - 1, Utot, NW);
           // With at least one unit per worker every worker in [wf, wl] holds
-          // part of the head, and only wf can hold it as its last head.
+          // part of the head; otherwise some ranges in it are empty.
           const bool dense = Utot >= NW;
           int last = 0;
           if (lane == 0) {
@@ -468,59 +565,36 @@ dmc_decode_kernel(const DecodeArgs a) {
           last = __shfl_sync(0xffffffffu, last, 0);
           if (last) {
             __threadfence();  // every contributor's partial is visible to this lane
-            constexpr int DPL = D / 32;  // output dims per lane
-            float Oc[DPL];
-#pragma unroll
-            for (int i = 0; i < DPL; ++i) Oc[i] = 0.f;
-            float Lc = 0.f;
-            if (dense && wl - wf < 32) {
-              // lane c reads contributor wf + c's (m, l); the dims are read in
-              // one pass of independent loads
-              const int nc = wl - wf + 1;
-              const int first_slot = (hu0 > range_start(wf, Utot, NW)) ? 1 : 0;
-              const int cs = 2 * (wf + lane) + (lane == 0 ? first_slot : 0);
-              float mc = -INFINITY, lc = 0.f;
-              if (lane < nc) {
-                mc = __ldcg(L.partials + (size_t)cs * (D + 2));
-                lc = __ldcg(L.partials + (size_t)cs * (D + 2) + 1);
-              }
-              float Mc = mc;
-#pragma unroll
-              for (int off = 16; off > 0; off >>= 1) Mc = fmaxf(Mc, __shfl_xor_sync(0xffffffffu, Mc, off));
-              const float wgt = (lane < nc && mc != -INFINITY) ? exp2f(mc - Mc) : 0.f;
-              Lc = lc * wgt;
-#pragma unroll
-              for (int off = 16; off > 0; off >>= 1) Lc += __shfl_xor_sync(0xffffffffu, Lc, off);
-              for (int c = 0; c < nc; ++c) {
-                const float w = __shfl_sync(0xffffffffu, wgt, c);
-                const int csc = __shfl_sync(0xffffffffu, cs, c);
-                const float* cp = L.partials + (size_t)csc * (D + 2) + 2 + lane * DPL;
-#pragma unroll
-                for (int i = 0; i < DPL; ++i) Oc[i] = fmaf(__ldcg(cp + i), w, Oc[i]);
-              }
+            if (dense) {
+              // worker wf + i wrote state 2 (wf + i) + 1 if the head starts
+              // inside its range (only possible for i = 0), else 2 (wf + i)
+              const int first_off = (hu0 > range_start(wf, Utot, NW)) ? 1 : 0;
+              combine_partials<T, D>(L.partials, wf, first_off, wl - wf + 1, lane, orow);
             } else {
-              float Mc = -INFINITY;
+              // fewer units than workers (tiny caches): one unit per non-empty
+              // range, so each contributor wrote state 2 cw of its range
+              float Mc = -INFINITY, Lc = 0.f;
               for (int cw = wf; cw <= wl; ++cw) {
-                const long long cs0 = range_start(cw, Utot, NW);
-                if (cs0 == range_start(cw + 1, Utot, NW)) continue;
-                const int cs = 2 * cw + (hu0 <= cs0 ? 0 : 1);
-                Mc = fmaxf(Mc, __ldcg(L.partials + (size_t)cs * (D + 2)));
+                if (range_start(cw, Utot, NW) == range_start(cw + 1, Utot, NW)) continue;
+                Mc = fmaxf(Mc, __ldcg(L.partials + (size_t)(2 * cw) * PSTRIDE));
               }
+              constexpr int DPL = D / 32;  // output dims per lane
+              float Oc[DPL];
+#pragma unroll
+              for (int i = 0; i < DPL; ++i) Oc[i] = 0.f;
               for (int cw = wf; cw <= wl; ++cw) {
-                const long long cs0 = range_start(cw, Utot, NW);
-                if (cs0 == range_start(cw + 1, Utot, NW)) continue;
-                const int cs = 2 * cw + (hu0 <= cs0 ? 0 : 1);
-                const float* cp = L.partials + (size_t)cs * (D + 2);
+                if (range_start(cw, Utot, NW) == range_start(cw + 1, Utot, NW)) continue;
+                const float* cp = L.partials + (size_t)(2 * cw) * PSTRIDE;
                 const float mc = __ldcg(cp);
                 const float cwt = (mc == -INFINITY) ? 0.f : exp2f(mc - Mc);
                 Lc = fmaf(__ldcg(cp + 1), cwt, Lc);
 #pragma unroll
-                for (int i = 0; i < DPL; ++i) Oc[i] = fmaf(__ldcg(cp + 2 + lane * DPL + i), cwt, Oc[i]);
+                for (int i = 0; i < DPL; ++i) Oc[i] = fmaf(__ldcg(cp + 4 + lane * DPL + i), cwt, Oc[i]);
               }
-            }
-            const float inv = 1.f / Lc;
+              const float inv = 1.f / Lc;
 #pragma unroll
-            for (int i = 0; i < DPL; ++i) orow[lane * DPL + i] = Elt<T>::from_f(Oc[i] * inv);
+              for (int i = 0; i < DPL; ++i) orow[lane * DPL + i] = Elt<T>::from_f(Oc[i] * inv);
+            }
           }
         }
         m = -INFINITY;
@@ -600,6 +674,7 @@ cudaError_t decode_setup(const Layout& L, int Gv, DecodePlan* plan) {
   const long long max_blocks = (max_units + kWarps - 1) / kWarps;
   if (e == cudaSuccess && max_blocks < plan->grid) plan->grid = (int)max_blocks;
   plan->partial_states = 2 * plan->grid * kWarps;
+  if (e == cudaSuccess && plan->partial_states > L.partial_cap) e = cudaErrorInvalidConfiguration;
   return e;
 }
 
@@ -642,9 +717,9 @@ cudaError_t decode_launch(const Layout& L, int layer, int Gv, const DecodePlan& 
 // ---------------------------------------------------------------- static scratch
 // Scratch of dmc_decode_step_static_scratch: room for the split-K partial
 // softmax states of one launch (2 per worker warp, head_dim <= 128, at most
-// 512 blocks of 8 warps), 4.26 MB. Every GPU that loads the library holds it
+// 512 blocks of 8 warps), 4.33 MB. Every GPU that loads the library holds it
 // until exit.
-constexpr size_t kStaticPartialFloats = (size_t)2 * kMaxWorkers * (128 + 2);
+constexpr size_t kStaticPartialFloats = (size_t)2 * kMaxWorkers * kPartialStride<128>;
 static __device__ __align__(256) float g_decode_static_partials[kStaticPartialFloats];
 
 // Host code must not pass g_decode_static_partials itself to a kernel (on the

@@ -33,8 +33,8 @@ struct Layout {
   float* pending_z;        // [NH]: their z
   unsigned long long* pool_top;
   unsigned int* error;
-  float* partials;         // [2 * max_blocks][D + 2]
-  int max_blocks;
+  float* partials;         // [partial_cap][D + 2]: split-K partial softmax states (m, l, acc)
+  int partial_cap;
   unsigned char* opens;    // [max_prefill_tokens][Hkv]: token opens a slot
   int* plan;               // [Hkv][plan_stride]: first slot index per prompt chunk
   int plan_stride;

@@ -49,6 +49,63 @@ def cache_for(wl: S.Workload, device, max_slots=None, num_pages=None, max_prefil
                     wl.torch_dtype, max_slots, num_pages, max_prefill_tokens, device=device)
 
 
+def exact_final_lengths(wl: S.Workload, device, steps, p=None):
+    """Slot count of every (layer, seq, kv head) after its prompt and `steps`
+    decode tokens, from the signs of the generated decision neurons. Used only
+    to size the page pool of the large workloads exactly; the parity checks
+    take their lengths from the oracle's rule."""
+    if p is None:
+        p = S.append_prob(wl)
+    out = torch.zeros((wl.num_layers, wl.batch, wl.num_kv_heads), dtype=torch.int64)
+    for layer in range(wl.num_layers):
+        pr = S.gen_prompt(wl, layer, device, p=p)
+        cu = pr["cu_seqlens"].to(torch.int64)
+        neg = (pr["k"][:, :, 0] < 0).to(torch.int64)
+        csum = torch.cat([torch.zeros_like(neg[:1]), torch.cumsum(neg, 0)])
+        n = csum[cu[1:]] - csum[cu[:-1]]
+        nonempty = (cu[1:] > cu[:-1])[:, None]
+        first_acc = (pr["k"][cu[:-1].clamp(max=max(int(cu[-1]) - 1, 0)), :, 0] >= 0) & nonempty
+        lens = n + first_acc.to(torch.int64)
+        del pr, neg, csum
+        for step in range(steps):
+            k0 = S.gen_decode(wl, layer, step, device, p=p)["k"][:, :, 0]
+            lens = lens + ((lens == 0) | (k0 < 0)).to(torch.int64)
+        out[layer] = lens.cpu()
+    return out
+
+
+def full_size_cache(wl: S.Workload, device, steps, margin_bytes=3 << 30):
+    """A cache for a full-size workload with an exactly sized page pool. If the
+    device cannot hold every layer next to one layer's prompt inputs, the
+    workload keeps its leading layers that fit (same per-layer shape, same
+    seeds); returns (workload, cache)."""
+    final = exact_final_lengths(wl, device, steps)
+    torch.cuda.empty_cache()
+    pages = ((final + 31) // 32).sum(dim=(1, 2)).cumsum(0)          # pages of layers [0, l]
+    lens = S.prompt_lengths(wl)
+    max_slots = int(final.max()) + 1
+    total = int(lens.sum())
+    row = wl.head_dim * wl.esize
+    # one layer's prompt in the cache dtype plus one sequence's fp32 draws
+    peak = total * (2 * wl.num_kv_heads * row + wl.num_q_heads * wl.esize) + \
+        int(lens.max()) * (3 * wl.num_kv_heads * wl.head_dim + wl.num_q_heads) * 4
+    free = torch.cuda.mem_get_info(device)[0]
+    from paper_2403_09636_gb300 import dmc_cache_config, dmc_cache_required_bytes, PAGE_SIZE
+    dt = 0 if wl.dtype == "f32" else 1
+    layers = wl.num_layers
+    while layers > 1:
+        cfg = dmc_cache_config(layers, wl.batch, wl.num_q_heads, wl.num_kv_heads, wl.head_dim, dt,
+                               PAGE_SIZE, max_slots, int(pages[layers - 1]) + 64, total, 0)
+        if dmc_cache_required_bytes(cfg) + peak + margin_bytes <= free:
+            break
+        layers -= 1
+    if layers < wl.num_layers:
+        wl = S.shrink(wl, num_layers=layers)
+    cache = cache_for(wl, device, max_slots=max_slots, num_pages=int(pages[layers - 1]) + 64,
+                      max_prefill_tokens=total)
+    return wl, cache
+
+
 class Run:
     """Prefill + decode of a workload on the GPU, keeping host copies of the
     inputs of sampled (layer, seq, kv_head) instances and the GPU results for
@@ -99,7 +156,12 @@ class Run:
             n = int(ln[0])
             self.prompt_export[s] = (k[0, :n].float().cpu().numpy(), v[0, :n].float().cpu().numpy(),
                                      z[0, :n].cpu().numpy(), n)
-        Hq = wl.num_q_heads
+        by_layer = {}
+        for s in self.samples:
+            by_layer.setdefault(s[0], []).append(s)
+        idx = {l: (torch.tensor([b for (_, b, _) in ss], device=device),
+                   torch.tensor([h for (_, _, h) in ss], device=device)) for l, ss in by_layer.items()}
+        B, Hkv = wl.batch, wl.num_kv_heads
         for step in range(steps):
             for layer in range(wl.num_layers):
                 dd = S.gen_decode(wl, layer, step, device, p=p)
@@ -112,15 +174,19 @@ class Run:
                         self.len_ok = False
                         self.len_msgs.append(f"step {step} layer {layer}: {np.argwhere(exp != got)[:5]}")
                     lens_now[layer] = exp
-                for s in self.samples:
-                    if s[0] != layer:
-                        continue
-                    _, b, h = s
+                if layer not in by_layer:
+                    continue
+                ib, ih = idx[layer]
+                kk = dd["k"][ib, ih].float().cpu().numpy()
+                vv = dd["v"][ib, ih].float().cpu().numpy()
+                qq = dd["q"].view(B, Hkv, G, d)[ib, ih].float().cpu().numpy()
+                oo = out.view(B, Hkv, G, d)[ib, ih].float().cpu().numpy()
+                for i, s in enumerate(by_layer[layer]):
                     I = self.inst[s]
-                    I["k_dec"].append(dd["k"][b, h].float().cpu().numpy())
-                    I["v_dec"].append(dd["v"][b, h].float().cpu().numpy())
-                    I["q_dec"].append(dd["q"][b, h * G:(h + 1) * G].float().cpu().numpy())
-                    I["out"].append(out[b, h * G:(h + 1) * G].float().cpu().numpy())
+                    I["k_dec"].append(kk[i])
+                    I["v_dec"].append(vv[i])
+                    I["q_dec"].append(qq[i])
+                    I["out"].append(oo[i])
         self.final_export = {}
         for s in self.samples:
             layer, b, h = s

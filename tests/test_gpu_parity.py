@@ -54,15 +54,6 @@ def test_f32_head_dim_128(cuda_dev):
     _check(H.Run(wl, cuda_dev, H.all_samples(wl)))
 
 
-def test_llama2_7b_4x_full_shape_sampled(cuda_dev):
-    """The benchmark workload itself (32 layers, batch 32, 32 heads, d 128,
-    prompt 2048, uniform 4x), lengths of every head of every layer after the
-    prompt and every decode step, slots and outputs of sampled heads. Decode
-    runs 64 of the 512 steps to keep the test short."""
-    wl = S.WORKLOADS["llama2_7b_4x"]
-    _check(H.Run(wl, cuda_dev, H.random_samples(wl, 48, seed=7), decode_steps=64))
-
-
 def test_gqa_virtual_heads_read_the_old_last_slot(cuda_dev):
     """Every query of a group merges the new token into the same old last
     slot; the group's one writer must not let another query see the merged
