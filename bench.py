@@ -57,6 +57,8 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--graph", action="store_true",
+                    help="replay the step's launches from CUDA graphs instead of launching from the host")
     return ap.parse_args()
 
 
@@ -101,6 +103,23 @@ def committed_traffic(workload, sources, per_launch_bytes):
     if j.get("source_sha") != decode_source_sha(sources):
         return None
     return per_launch_bytes * j["captured_dram_bytes"] / j["captured_algorithmic_bytes"]
+
+
+def max_over_ranks(dist, values, device):
+    """Each rank's timings -> the element-wise maximum over all ranks (the
+    slowest replica sets the job's time). `dist` None means one process."""
+    if dist is None:
+        return list(values)
+    import torch
+    t = torch.tensor(list(values), device=device, dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return t.tolist()
+
+
+def job_rate(world, steps, tokens_per_step, ms):
+    """Whole-job throughput: every replica processes `tokens_per_step` in each
+    of `steps` steps; `ms` is the slowest replica's time."""
+    return world * steps * tokens_per_step / (ms / 1e3)
 
 
 class ClockSampler:
@@ -298,22 +317,39 @@ def run_ours(args, rank, world, dist):
     h = cache.handle
     pf_fn, dec_fn, reset_fn = L_.dmc_prefill_compress, L_.dmc_decode_step, L_.dmc_cache_reset
 
-    def one_step(ev=None):
+    def prefill_all(sh):
         rc = reset_fn(h, sh)
-        if ev is not None:
-            ev[0].record(stream)
         for l, (q0, s0, s1, kp, vp, cu, tot, mx, ns) in enumerate(qp):
             rc |= pf_fn(h, l, 0, ns, q0, s0, s1, kp, vp, cu, tot, mx, sh)
-        if ev is not None:
-            ev[1].record(stream)
+        if rc:
+            raise RuntimeError(f"launch failed: {rc}")
+
+    def decode_all(sh):
+        rc = 0
         for t in range(steps_dec):
             for l in range(Lr):
                 a = dptr[t][l]
                 rc |= dec_fn(h, l, a[0], a[1], a[2], a[3], sh)
-        if ev is not None:
-            ev[2].record(stream)
         if rc:
             raise RuntimeError(f"launch failed: {rc}")
+
+    graphs = None
+
+    def one_step(ev=None):
+        if ev is not None:
+            ev[0].record(stream)
+        if graphs is None:
+            prefill_all(sh)
+        else:
+            graphs[0].replay()
+        if ev is not None:
+            ev[1].record(stream)
+        if graphs is None:
+            decode_all(sh)
+        else:
+            graphs[1].replay()
+        if ev is not None:
+            ev[2].record(stream)
 
     def barrier():
         torch.cuda.synchronize()
@@ -329,6 +365,21 @@ def run_ours(args, rank, world, dist):
     got = torch.stack([cache.lengths(l) for l in range(Lr)])
     if not torch.equal(got.to(torch.int64), final):
         raise RuntimeError("slot counts after a step differ from the decisions")
+    if args.graph:
+        # the step's launch sequence captured once: reset + prefill, then every
+        # decode launch (programmatic dependencies between decodes are kept)
+        torch.cuda.synchronize()
+        graphs = [torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()]
+        with torch.cuda.graph(graphs[0]):
+            prefill_all(torch.cuda.current_stream().cuda_stream)
+        with torch.cuda.graph(graphs[1]):
+            decode_all(torch.cuda.current_stream().cuda_stream)
+        torch.cuda.synchronize()
+        for _ in range(max(1, args.warmup)):
+            one_step()
+        got = torch.stack([cache.lengths(l) for l in range(Lr)])
+        if not torch.equal(got.to(torch.int64), final):
+            raise RuntimeError("slot counts after a graph step differ from the decisions")
 
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -345,14 +396,10 @@ def run_ours(args, rank, world, dist):
     st, bits, _ = cache.status()
     if st != 0:
         raise RuntimeError(f"device fault in timed region: status {st} bits {bits:#x}")
-    if dist is not None:
-        t = torch.tensor([total_ms, pf_ms, dec_ms], device=dev, dtype=torch.float64)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms, pf_ms, dec_ms = t.tolist()
+    total_ms, pf_ms, dec_ms = max_over_ranks(dist, [total_ms, pf_ms, dec_ms], dev)
 
     K = args.steps
-    gen_tokens = world * K * Bt * steps_dec
-    value = gen_tokens / (total_ms / 1e3)
+    value = job_rate(world, K, Bt * steps_dec, total_ms)
     avg_launch_s = dec_ms / 1e3 / (K * n_dec_launch)
     per_launch_bytes = dec_bytes / n_dec_launch
     achieved = per_launch_bytes / avg_launch_s / 1e9
@@ -368,10 +415,11 @@ def run_ours(args, rank, world, dist):
                    "decode_steps": steps_dec, "cr": list(wl.cr), "page_size": 32,
                    "global_batch": Bt * world, "seq_len": int(S.prompt_lengths(wl).max()) + steps_dec,
                    "parallelism": f"replicas{world}",
+                   "launch": "cuda_graph" if args.graph else "stream",
                    "l2": "inputs larger than L2: each decode launch streams ~"
                          f"{per_launch_bytes / 1e6:.0f} MB of slots, layers rotate"},
-        "decode_only_tokens_per_s": world * K * Bt * steps_dec / (dec_ms / 1e3),
-        "prefill_tokens_per_s": world * K * pf_tokens / (pf_ms / 1e3),
+        "decode_only_tokens_per_s": job_rate(world, K, Bt * steps_dec, dec_ms),
+        "prefill_tokens_per_s": job_rate(world, K, pf_tokens, pf_ms),
         "decode_hbm_gbs": achieved,
         "decode_frac_of_8tbs": achieved / NOMINAL_HBM_GBS,
         "prefill_hbm_gbs": K * pf_bytes / (pf_ms / 1e3) / 1e9,
@@ -455,15 +503,11 @@ def run_e2e(args, wl, cache, prompts, qd, kd, vd, outs, steps_dec, dev, stream, 
         step()
     e1.record(stream)
     barrier()
-    ms = e0.elapsed_time(e1)
-    if dist is not None:
-        t = torch.tensor([ms], device=dev, dtype=torch.float64)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = t.item()
+    ms = max_over_ranks(dist, [e0.elapsed_time(e1)], dev)[0]
     st, bits, _ = cache.status()
     if st != 0:
         raise RuntimeError(f"device fault in e2e: status {st} bits {bits:#x}")
-    return {"value": world * args.steps * wl.batch * steps_dec / (ms / 1e3), "unit": "tokens/s",
+    return {"value": job_rate(world, args.steps, wl.batch * steps_dec, ms), "unit": "tokens/s",
             "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
             "note": f"pinned host inputs: one layer's prompt reused for all {Lr} layers, a ring of "
                     f"{ring} decode steps reused cyclically; every attention output is read back into a "
