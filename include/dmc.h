@@ -119,6 +119,33 @@ dmc_status dmc_prefill_compress(dmc_cache_t cache, int32_t layer, int32_t first_
                                 const int32_t* cu_seqlens_dev, int32_t total_tokens,
                                 int32_t max_seqlen, cudaStream_t stream);
 
+/* dmc_prefill_compress plus the attention output of every prompt token.
+ * At inference a prompt token attends over the cache as it stands right after
+ * its own update (Eq. attn-softmax over the compressed slots; the training
+ * mask of Sec. 3.2 with binary alpha gives the same pattern): the final values
+ * of the slots closed before it, and the slot it has just merged into or
+ * opened, whose value at that moment is the running omega-weighted mean of its
+ * segment (Eq. partial-accumulation). The cache afterwards is exactly as after
+ * dmc_prefill_compress of the same prompt; a head that already holds slots
+ * continues its last segment, so splitting a prompt over calls gives the same
+ * outputs. The score is q[1:]^T k[1:] / sqrt(head_dim) (q[0] and k[0] are the
+ * gates). Runs on the tcgen05 tensor cores: bf16 caches with head_dim 128 and
+ * 1, 2, 4 or 8 query heads per KV head; other caches return
+ * DMC_ERR_INVALID_ARG.
+ *   q_dev:   [total_tokens, num_q_heads, head_dim], packed (q[., ., 0] also
+ *            gives omega, as in dmc_prefill_compress);
+ *   k_dev, v_dev: [total_tokens, num_kv_heads, head_dim], sequences packed;
+ *   cu_seqlens_dev, total_tokens, max_seqlen: as in dmc_prefill_compress;
+ *   out_dev: [total_tokens, num_q_heads, head_dim] (written, bf16).
+ * All device pointers 16-byte aligned. Asynchronous on `stream`; device faults
+ * (capacity, pool, bad cu_seqlens, a wait that gave up) set the sticky bits
+ * read by dmc_cache_status. */
+dmc_status dmc_prefill_attention(dmc_cache_t cache, int32_t layer, int32_t first_seq,
+                                 int32_t num_seqs, const void* q_dev, const void* k_dev,
+                                 const void* v_dev, const int32_t* cu_seqlens_dev,
+                                 int32_t total_tokens, int32_t max_seqlen, void* out_dev,
+                                 cudaStream_t stream);
+
 /* One decode step of one layer for all `batch` sequences: Algorithm 1 on the
  * new token of every KV head (append or accumulate, fused), then every query
  * head attends over its KV head's updated slots (split across thread blocks
@@ -139,7 +166,7 @@ dmc_status dmc_decode_step(dmc_cache_t cache, int32_t layer, const void* q_dev,
  * implicit device synchronisation. Same arguments, semantics and results as
  * dmc_decode_step; it allocates nothing and calls no allocating routine.
  * The scratch is the split-K partial softmax states of one launch, kept in a
- * file-scope __device__ array of 4.26 MB (2 states of head_dim + 2 floats for
+ * file-scope __device__ array of 4.33 MB (2 states of head_dim + 4 floats for
  * each of at most 4096 worker warps) that every GPU loading the library holds
  * until the process exits; a cache whose decode grid would need more returns
  * DMC_ERR_INVALID_ARG. Nothing in it needs to start at zero: each launch writes

@@ -161,6 +161,22 @@ def run_head(k_prompt, v_prompt, q0_prompt, k_dec, v_dec, q_dec, cache=None):
             "cache": cache}
 
 
+def prompt_attention(k, v, q, cache=None):
+    """Attention outputs of every prompt token at inference (formulation A).
+
+    Sec. 3.2 (intermediate compression steps): at inference the last slot
+    changes in place, so each prompt token sees the cache as it stands after
+    its own update: the closed slots and its segment's running state. That is
+    the decode step applied to the prompt tokens one by one (Algorithm 1, then
+    Eq. attn-softmax), which is what this returns; `masked_attention` is the
+    training-time statement of the same thing. k, v [T, d]; q [T, G, d]; an
+    existing `cache` is continued. Returns [T, G, d]."""
+    d = np.asarray(k).shape[1]
+    G = np.asarray(q).shape[1]
+    empty = np.zeros((0, d))
+    return run_head(empty, empty, np.zeros((0, G)), k, v, q, cache=cache)["out"]
+
+
 def decode_lengths(k0_tokens, start_len: int = 0) -> np.ndarray:
     """Cache length after each token, from the decisions alone (Sec. 3.1:
     l = sum_t (1 - alpha_t), with an empty cache's first token always opening

@@ -30,7 +30,7 @@ DMC_FAULT_WAIT_TIMEOUT = 0x10
 PAGE_SIZE = 32
 
 EXPORTED = ("dmc_cache_required_bytes", "dmc_cache_create", "dmc_cache_destroy",
-            "dmc_cache_reset", "dmc_prefill_compress", "dmc_decode_step",
+            "dmc_cache_reset", "dmc_prefill_compress", "dmc_prefill_attention", "dmc_decode_step",
             "dmc_decode_step_static_scratch", "dmc_cache_lengths",
             "dmc_cache_export_heads", "dmc_cache_status", "dmc_status_string")
 
@@ -70,6 +70,7 @@ def lib():
             "dmc_cache_reset": (C.c_int, [vp, vp]),
             "dmc_prefill_compress": (C.c_int, [vp, i32, i32, i32, vp, i64, i64, vp, vp, vp, i32,
                                                i32, vp]),
+            "dmc_prefill_attention": (C.c_int, [vp, i32, i32, i32, vp, vp, vp, vp, i32, i32, vp, vp]),
             "dmc_decode_step": (C.c_int, [vp, i32, vp, vp, vp, vp, vp]),
             "dmc_decode_step_static_scratch": (C.c_int, [vp, i32, vp, vp, vp, vp, vp]),
             "dmc_cache_lengths": (C.c_int, [vp, i32, vp, vp]),
@@ -111,6 +112,12 @@ def dmc_prefill_compress(handle, layer, first_seq, num_seqs, q_ptr, q_token_stri
     return lib().dmc_prefill_compress(handle, layer, first_seq, num_seqs, q_ptr, q_token_stride,
                                       q_head_stride, k_ptr, v_ptr, cu_seqlens_ptr, total_tokens,
                                       max_seqlen, stream)
+
+
+def dmc_prefill_attention(handle, layer, first_seq, num_seqs, q_ptr, k_ptr, v_ptr, cu_seqlens_ptr,
+                          total_tokens, max_seqlen, out_ptr, stream) -> int:
+    return lib().dmc_prefill_attention(handle, layer, first_seq, num_seqs, q_ptr, k_ptr, v_ptr,
+                                       cu_seqlens_ptr, total_tokens, max_seqlen, out_ptr, stream)
 
 
 def dmc_decode_step(handle, layer, q_ptr, k_ptr, v_ptr, out_ptr, stream) -> int:
@@ -202,6 +209,15 @@ class DmcCache:
                                     q0.stride(0), q0.stride(1), k.data_ptr(), v.data_ptr(),
                                     cu_seqlens.data_ptr(), total, int(max_seqlen),
                                     self._s(stream)), "dmc_prefill_compress")
+
+    def prefill_attention(self, layer, q, k, v, cu_seqlens, max_seqlen, out, first_seq=0,
+                          stream=None):
+        """q, out: [total, Hq, D]; k, v: [total, Hkv, D]; cu_seqlens int32."""
+        n = cu_seqlens.numel() - 1
+        _check(dmc_prefill_attention(self.handle, layer, first_seq, n, q.data_ptr(), k.data_ptr(),
+                                     v.data_ptr(), cu_seqlens.data_ptr(), k.shape[0],
+                                     int(max_seqlen), out.data_ptr(), self._s(stream)),
+               "dmc_prefill_attention")
 
     def decode(self, layer, q, k, v, out, stream=None):
         _check(dmc_decode_step(self.handle, layer, q.data_ptr(), k.data_ptr(), v.data_ptr(),

@@ -15,7 +15,13 @@ cudaError_t decode_launch(const Layout& L, int layer, int Gv, const DecodePlan& 
                           cudaStream_t stream);
 cudaError_t prefill_launch(const Layout& L, int layer, int first_seq, int num_seqs, const void* q,
                            long long q_tok, long long q_head, const void* k, const void* v,
-                           const int* cu, int total_tokens, int max_seqlen, cudaStream_t stream);
+                           const int* cu, int total_tokens, int max_seqlen, float* carry,
+                           cudaStream_t stream);
+bool prefill_attn_supported(const Layout& L);
+cudaError_t prefill_attn_launch(const Layout& L, int layer, int first_seq, int num_seqs,
+                                const void* q, const void* k, const void* v, const int* cu,
+                                int total_tokens, int max_seqlen, const float* carry, void* out,
+                                cudaStream_t stream);
 cudaError_t decode_static_partials(int device, float** ptr, size_t* floats);
 bool gqa_supported(const Layout& L);
 cudaError_t gqa_setup(const Layout& L, DecodePlan* plan);
@@ -40,6 +46,7 @@ struct dmc_cache {
   int last_decode_layer;  // layer of the latest kernel if it was a decode, else -1
   char* meta;  // lengths, ctl, counters, pool top, error: cleared by create / reset
   size_t meta_bytes;
+  float* carry;  // segment sums at prompt chunk starts (prompt attention)
 };
 
 namespace {
@@ -67,7 +74,7 @@ bool valid_config(const dmc_cache_config* c) {
 // Byte offsets of every region; returns the total size.
 struct Offsets {
   size_t pages, z, ptab, meta, lengths, ctl, counters, pool_top, error, meta_end, partials,
-      pending, pending_at, pending_z, opens, plan, total;
+      pending, pending_at, pending_z, opens, plan, carry, total;
   int MPH, plan_stride;
 };
 
@@ -97,6 +104,7 @@ Offsets offsets(const dmc_cache_config* c) {
   o.pending_z = at; at = align_up(at + (G > 1 ? (size_t)NH * 4 : 0));
   o.opens = at; at = align_up(at + (size_t)c->max_prefill_tokens * c->num_kv_heads);
   o.plan = at; at = align_up(at + (size_t)c->num_kv_heads * o.plan_stride * 4);
+  o.carry = at; at = align_up(at + (size_t)o.plan_stride * c->num_kv_heads * (2 * c->head_dim + 1) * 4);
   o.total = at;
   return o;
 }
@@ -191,6 +199,7 @@ dmc_status dmc_cache_create(const dmc_cache_config* cfg, void* arena_dev, size_t
   L.opens = reinterpret_cast<unsigned char*>(base + o.opens);
   L.plan = reinterpret_cast<int*>(base + o.plan);
   L.plan_stride = o.plan_stride;
+  c->carry = reinterpret_cast<float*>(base + o.carry);
   L.max_prefill_tokens = cfg->max_prefill_tokens;
   c->meta = base + o.meta;
   c->meta_bytes = o.meta_end - o.meta;
@@ -250,7 +259,35 @@ dmc_status dmc_prefill_compress(dmc_cache_t c, int32_t layer, int32_t first_seq,
   c->last_decode_layer = -1;
   return cuda_status(dmc::prefill_launch(L, layer, first_seq, num_seqs, q_dev, q_token_stride,
                                          q_head_stride, k_dev, v_dev, cu_seqlens_dev, total_tokens,
-                                         max_seqlen, stream));
+                                         max_seqlen, nullptr, stream));
+}
+
+dmc_status dmc_prefill_attention(dmc_cache_t c, int32_t layer, int32_t first_seq,
+                                 int32_t num_seqs, const void* q_dev, const void* k_dev,
+                                 const void* v_dev, const int32_t* cu_seqlens_dev,
+                                 int32_t total_tokens, int32_t max_seqlen, void* out_dev,
+                                 cudaStream_t stream) {
+  if (!c) return DMC_ERR_INVALID_ARG;
+  const Layout& L = c->lay;
+  if (!dmc::prefill_attn_supported(L)) return DMC_ERR_INVALID_ARG;
+  if (layer < 0 || layer >= L.L || first_seq < 0 || num_seqs < 0 || first_seq + num_seqs > L.B)
+    return DMC_ERR_INVALID_ARG;
+  if (total_tokens < 0 || total_tokens > L.max_prefill_tokens || max_seqlen < 0 ||
+      max_seqlen > total_tokens)
+    return DMC_ERR_INVALID_ARG;
+  if (num_seqs == 0 || total_tokens == 0) return DMC_OK;
+  if (!q_dev || !k_dev || !v_dev || !cu_seqlens_dev || !out_dev || !aligned16(q_dev) ||
+      !aligned16(k_dev) || !aligned16(v_dev) || !aligned16(out_dev))
+    return DMC_ERR_INVALID_ARG;
+  c->last_decode_layer = -1;
+  const long long q_tok = (long long)L.Hq * L.D, q_head = L.D;
+  cudaError_t e = dmc::prefill_launch(L, layer, first_seq, num_seqs, q_dev, q_tok, q_head, k_dev,
+                                      v_dev, cu_seqlens_dev, total_tokens, max_seqlen, c->carry,
+                                      stream);
+  if (e != cudaSuccess) return DMC_ERR_CUDA;
+  return cuda_status(dmc::prefill_attn_launch(L, layer, first_seq, num_seqs, q_dev, k_dev, v_dev,
+                                              cu_seqlens_dev, total_tokens, max_seqlen, c->carry,
+                                              out_dev, stream));
 }
 
 dmc_status dmc_decode_step(dmc_cache_t c, int32_t layer, const void* q_dev, const void* k_dev,

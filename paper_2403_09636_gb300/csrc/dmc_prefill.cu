@@ -16,7 +16,11 @@
 //        the chunk end is followed to its end, so each k/v row is read once.
 //        Warps take segments round-robin; lanes split a row into 16-byte pieces
 //        and accumulate sum(omega k), sum(omega v), sum(omega) in fp32; the slot
-//        is the quotient, rounded once to the cache dtype.
+//        is the quotient, rounded once to the cache dtype. When asked for
+//        (prompt attention), the block also records, at every chunk start a
+//        segment runs across, the segment's sums up to that point (the
+//        "carry"), so that each chunk can rebuild the running state of its
+//        tokens without reading back to the segment's start.
 #include "dmc_internal.cuh"
 
 namespace dmc {
@@ -33,6 +37,7 @@ struct PrefillArgs {
   const char* v;
   const int* cu;
   int total_tokens, max_seqlen;
+  float* carry;  // [chunk id][Hkv][2D + 1] (sum w k, sum w v, sum w), or null
 };
 
 __device__ __forceinline__ bool seq_bounds(const PrefillArgs& a, int s, int& t0, int& t1) {
@@ -136,9 +141,15 @@ __global__ void __launch_bounds__(kPlanThreads) dmc_prefill_plan_kernel(const Pr
   }
 }
 
+// Carry slot of the chunk of sequence s that starts at token cs (t0 = the
+// sequence's first token).
+__device__ __forceinline__ float* carry_at(const PrefillArgs& a, int t0, int cs, int s, int h, int D) {
+  return a.carry + ((size_t)chunk_id(t0, (cs - t0) / kPrefillChunk, s) * a.lay.Hkv + h) * (2 * D + 1);
+}
+
 template <typename T, int D>
 __device__ __forceinline__ void scan_segment(const PrefillArgs& a, int h, int bh, int tb, int te,
-                                             int slot, bool merge_old) {
+                                             int slot, bool merge_old, int t0, int s) {
   using CK = Chunk<T>;
   constexpr int ROW = D * (int)sizeof(T);
   constexpr int LPR = ROW / 16;  // lanes per row
@@ -150,27 +161,84 @@ __device__ __forceinline__ void scan_segment(const PrefillArgs& a, int h, int bh
   float ak[EPC], av[EPC], zs = 0.f;
 #pragma unroll
   for (int e = 0; e < EPC; ++e) { ak[e] = 0.f; av[e] = 0.f; }
+  const int page = L.page_table[((size_t)a.layer * L.NH + bh) * L.MPH + slot / kPage];
+  char* kdst = L.pages + (size_t)page * L.page_bytes + (size_t)(slot % kPage) * ROW + lr * 16;
+  char* vdst = kdst + (size_t)kPage * ROW;
+  float* zp = L.z + (size_t)page * kPage + slot % kPage;
+  if (merge_old && sub == 0) {
+    // the prompt continues the head's last slot: its K z_old, V z_old and
+    // z_old join the sums (one copy, in the first row group's lanes)
+    float ko[EPC], vo[EPC];
+    CK::unpack(*reinterpret_cast<const uint4*>(kdst), ko);
+    CK::unpack(*reinterpret_cast<const uint4*>(vdst), vo);
+    const float zo = *zp;
+#pragma unroll
+    for (int e = 0; e < EPC; ++e) {
+      ak[e] = ko[e] * zo;
+      av[e] = vo[e] * zo;
+    }
+    zs = lr == 0 ? zo : 0.f;
+  }
+  // Writes the sums so far (all row groups together) as the carry of the chunk
+  // starting at token cs.
+  auto put_carry = [&](int cs) {
+    float sk[EPC], sv[EPC];
+    float sz = zs;
+#pragma unroll
+    for (int e = 0; e < EPC; ++e) { sk[e] = ak[e]; sv[e] = av[e]; }
+#pragma unroll
+    for (int off = LPR; off < 32; off <<= 1) {
+#pragma unroll
+      for (int e = 0; e < EPC; ++e) {
+        sk[e] += __shfl_xor_sync(0xffffffffu, sk[e], off);
+        sv[e] += __shfl_xor_sync(0xffffffffu, sv[e], off);
+      }
+      sz += __shfl_xor_sync(0xffffffffu, sz, off);
+    }
+    if (sub == 0) {
+      float* cp = carry_at(a, t0, cs, s, h, D);
+#pragma unroll
+      for (int e = 0; e < EPC; ++e) {
+        cp[lr * EPC + e] = sk[e];
+        cp[D + lr * EPC + e] = sv[e];
+      }
+      if (lr == 0) cp[2 * D] = sz;
+    }
+  };
+  const bool carry = a.carry != nullptr;
+  if (carry && merge_old) put_carry(t0);  // the state the prompt's first token continues
   const size_t hrow = (size_t)L.Hkv * ROW;
   const char* kb = a.k + (size_t)h * ROW + lr * 16;
   const char* vb = a.v + (size_t)h * ROW + lr * 16;
-#pragma unroll 2
-  for (int t = tb + sub; t < te; t += RPI) {
-    const uint4 kr = __ldg(reinterpret_cast<const uint4*>(kb + (size_t)t * hrow));
-    const uint4 vr = __ldg(reinterpret_cast<const uint4*>(vb + (size_t)t * hrow));
-    float y = 0.f;
-    for (int g = 0; g < L.G; ++g)
-      y += Elt<T>::to_f(qq[(size_t)t * a.q_tok + (size_t)(h * L.G + g) * a.q_head]);
-    const float w = sigmoidf_(y / (float)L.G);  // omega = sigmoid(q[0]) (group mean for GQA)
-    float kf[EPC], vf[EPC];
-    CK::unpack(kr, kf);
-    CK::unpack(vr, vf);
-    if (lr == 0) kf[0] = 0.f;  // k[0] <- 0 (Algorithm 1)
-#pragma unroll
-    for (int e = 0; e < EPC; ++e) {
-      ak[e] = fmaf(w, kf[e], ak[e]);
-      av[e] = fmaf(w, vf[e], av[e]);
+  // the segment in pieces that end at chunk starts (only split when carries are asked for)
+  int pb = tb;
+  while (pb < te) {
+    int pe = te;
+    if (carry) {
+      const int next_chunk = t0 + ((pb - t0) / kPrefillChunk + 1) * kPrefillChunk;
+      pe = min(te, next_chunk);
     }
-    zs += w;
+#pragma unroll 2
+    for (int t = pb + sub; t < pe; t += RPI) {
+      const uint4 kr = __ldg(reinterpret_cast<const uint4*>(kb + (size_t)t * hrow));
+      const uint4 vr = __ldg(reinterpret_cast<const uint4*>(vb + (size_t)t * hrow));
+      float y = 0.f;
+      for (int g = 0; g < L.G; ++g)
+        y += Elt<T>::to_f(qq[(size_t)t * a.q_tok + (size_t)(h * L.G + g) * a.q_head]);
+      const float w = sigmoidf_(y / (float)L.G);  // omega = sigmoid(q[0]) (group mean for GQA)
+      float kf[EPC], vf[EPC];
+      CK::unpack(kr, kf);
+      CK::unpack(vr, vf);
+      if (lr == 0) kf[0] = 0.f;  // k[0] <- 0 (Algorithm 1)
+#pragma unroll
+      for (int e = 0; e < EPC; ++e) {
+        ak[e] = fmaf(w, kf[e], ak[e]);
+        av[e] = fmaf(w, vf[e], av[e]);
+      }
+      zs += w;
+    }
+    if (pe < te) put_carry(pe);  // the segment runs across the chunk starting at pe
+    pb = pe;
   }
 #pragma unroll
   for (int off = LPR; off < 32; off <<= 1) {
@@ -181,36 +249,19 @@ __device__ __forceinline__ void scan_segment(const PrefillArgs& a, int h, int bh
     }
     zs += __shfl_xor_sync(0xffffffffu, zs, off);
   }
+  // the lr == 0 lane holds z; every lane needs it for the quotient
+  zs = __shfl_sync(0xffffffffu, zs, lane - lr);
   if (sub != 0) return;
-  const int page = L.page_table[((size_t)a.layer * L.NH + bh) * L.MPH + slot / kPage];
-  char* kdst = L.pages + (size_t)page * L.page_bytes + (size_t)(slot % kPage) * ROW + lr * 16;
-  char* vdst = kdst + (size_t)kPage * ROW;
-  float* zp = L.z + (size_t)page * kPage + slot % kPage;
-  float kn[EPC], vn[EPC], znew;
-  if (merge_old) {
-    // the prompt continues the head's last slot: (K z_old + sum w k) / (z_old + sum w)
-    float ko[EPC], vo[EPC];
-    CK::unpack(*reinterpret_cast<const uint4*>(kdst), ko);
-    CK::unpack(*reinterpret_cast<const uint4*>(vdst), vo);
-    const float zo = *zp;
-    znew = zo + zs;
+  float kn[EPC], vn[EPC];
 #pragma unroll
-    for (int e = 0; e < EPC; ++e) {
-      kn[e] = (ko[e] * zo + ak[e]) / znew;
-      vn[e] = (vo[e] * zo + av[e]) / znew;
-    }
-  } else {
-    znew = zs;
-#pragma unroll
-    for (int e = 0; e < EPC; ++e) {
-      kn[e] = ak[e] / zs;
-      vn[e] = av[e] / zs;
-    }
+  for (int e = 0; e < EPC; ++e) {
+    kn[e] = ak[e] / zs;
+    vn[e] = av[e] / zs;
   }
   if (lr == 0) kn[0] = 0.f;
   *reinterpret_cast<uint4*>(kdst) = CK::pack(kn);
   *reinterpret_cast<uint4*>(vdst) = CK::pack(vn);
-  if (lr == 0) *zp = znew;
+  if (lr == 0) *zp = zs;
 }
 
 template <typename T, int D>
@@ -259,12 +310,12 @@ __global__ void __launch_bounds__(kScanThreads) dmc_prefill_scan_kernel(const Pr
   for (int it = warp; it < items; it += kScanThreads / 32) {
     if (pre && it == 0) {
       const int te = nstart > 0 ? starts[0] : next;
-      scan_segment<T, D>(a, h, bh, t0, te, base - 1, true);
+      scan_segment<T, D>(a, h, bh, t0, te, base - 1, true, t0, s);
     } else {
       const int j = it - (pre ? 1 : 0);
       const int tb = starts[j];
       const int te = (j + 1 < nstart) ? starts[j + 1] : next;
-      scan_segment<T, D>(a, h, bh, tb, te, base + j, false);
+      scan_segment<T, D>(a, h, bh, tb, te, base + j, false, t0, s);
     }
   }
 }
@@ -290,7 +341,8 @@ static cudaError_t launch_prefill(const PrefillArgs& a, cudaStream_t stream) {
 
 cudaError_t prefill_launch(const Layout& L, int layer, int first_seq, int num_seqs, const void* q,
                            long long q_tok, long long q_head, const void* k, const void* v,
-                           const int* cu, int total_tokens, int max_seqlen, cudaStream_t stream) {
+                           const int* cu, int total_tokens, int max_seqlen, float* carry,
+                           cudaStream_t stream) {
   PrefillArgs a;
   a.lay = L;
   a.layer = layer;
@@ -304,6 +356,7 @@ cudaError_t prefill_launch(const Layout& L, int layer, int first_seq, int num_se
   a.cu = cu;
   a.total_tokens = total_tokens;
   a.max_seqlen = max_seqlen;
+  a.carry = carry;
   if (L.esize == 4 && L.D == 64) return launch_prefill<float, 64>(a, stream);
   if (L.esize == 4 && L.D == 128) return launch_prefill<float, 128>(a, stream);
   if (L.esize == 2 && L.D == 64) return launch_prefill<__nv_bfloat16, 64>(a, stream);

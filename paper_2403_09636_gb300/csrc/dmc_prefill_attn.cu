@@ -1,0 +1,498 @@
+// Prompt-phase DMC attention on the fifth-generation tensor cores (tcgen05).
+//
+// At inference every prompt token attends over the cache as it stands right
+// after that token's own update (Eq. attn-softmax; the training mask of
+// Sec. 3.2 with binary alpha gives the same pattern): the slots closed before
+// the token, plus the slot the token has just merged into or opened, whose
+// value at that moment is the running omega-weighted mean of its segment so
+// far (Eq. partial-accumulation). With len(i) the slot count after token i,
+// query i therefore sees the final values of slots [0, len(i) - 1) and one
+// "diagonal" state.
+//
+// One CTA of 4 warps per (128 query rows, KV head, sequence); a row is a
+// (token, query head of the group) pair, token-major, so a group of G queries
+// shares every K/V tile. The closed slots are read from the cache pages that
+// the prefill scan has just written, in tiles of 128 slots:
+//   S = Q K^T          tcgen05.mma kind::f16, M = N = 128, K = head_dim, into TMEM
+//   softmax            one thread per row: tcgen05.ld of its S row, the
+//                      staircase mask (slot < len(i) - 1), online softmax in
+//                      the log2 domain, P rounded to bf16 into shared memory
+//   O += P V           tcgen05.mma with V as an MN-major B operand, into TMEM
+// The diagonal state of each token is rebuilt at the end from the prompt's
+// k, v rows of the token's 128-token chunk and the segment sums the prefill
+// scan recorded at the chunk start ("carry"), then merged into the row.
+#include <math.h>
+
+#include "dmc_internal.cuh"
+
+namespace dmc {
+
+constexpr int kPaRows = 128;     // query rows per tile (M)
+constexpr int kPaSlots = 128;    // slots per K/V tile (N of S, K of P V)
+constexpr int kPaThreads = 128;  // one thread per query row
+constexpr int kPaD = 128;        // head_dim handled by this kernel
+constexpr int kPaTileBytes = kPaRows * kPaD * 2;  // 32 KB: [128 rows][256 B]
+// dynamic shared memory: Q | K0 | K1 | V0 | V1 | P | misc
+constexpr int kPaQ = 0, kPaK = kPaTileBytes, kPaV = 3 * kPaTileBytes, kPaP = 5 * kPaTileBytes;
+constexpr int kPaMisc = 6 * kPaTileBytes;
+constexpr int kPaSmem = kPaMisc + 2048;
+
+struct PrefillAttnArgs {
+  Layout lay;
+  int layer, first_seq, num_seqs;
+  const char* q;   // [total_tokens][Hq][D]
+  const char* k;   // [total_tokens][Hkv][D]
+  const char* v;
+  const int* cu;
+  int total_tokens, max_seqlen;
+  const float* carry;  // [chunk id][Hkv][2D + 1]
+  char* out;           // [total_tokens][Hq][D]
+};
+
+// byte offset of 16-byte chunk j (0..15) of row r in a [128 rows][256 B] tile
+// kept as two 128-byte column halves, 128B-swizzled (chunk ^ row % 8)
+__device__ __forceinline__ uint32_t pa_swz(int r, int j) {
+  return (uint32_t)((j >> 3) * (kPaRows * 128) + r * 128 + (((j & 7) ^ (r & 7)) << 4));
+}
+
+// tcgen05 shared-memory matrix descriptor: 128B swizzle, start address, leading
+// and stride byte offsets (all in 16-byte units), descriptor version 1
+__device__ __forceinline__ uint64_t pa_desc(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+  return (uint64_t)((saddr >> 4) & 0x3FFF) | ((uint64_t)((lbo >> 4) & 0x3FFF) << 16) |
+         ((uint64_t)((sbo >> 4) & 0x3FFF) << 32) | ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
+}
+
+// instruction descriptor, kind::f16: bf16 A and B, fp32 D, M = N = 128;
+// b_mn selects an MN-major B operand
+__device__ __forceinline__ uint32_t pa_idesc(bool b_mn) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((b_mn ? 1u : 0u) << 16) | ((128u >> 3) << 17) |
+         ((128u >> 4) << 24);
+}
+
+__device__ __forceinline__ void pa_mma(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
+                                       bool acc) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(a), "l"(b), "r"(idesc), "r"(acc ? 1 : 0));
+}
+
+__device__ __forceinline__ void pa_commit(uint32_t bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+                   bar)
+               : "memory");
+}
+
+// 32 consecutive fp32 columns of this thread's TMEM lane
+__device__ __forceinline__ void pa_ld32(uint32_t taddr, float* f) {
+  uint32_t v[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,"
+      "%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+      : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]),
+        "=r"(v[7]), "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]),
+        "=r"(v[14]), "=r"(v[15]), "=r"(v[16]), "=r"(v[17]), "=r"(v[18]), "=r"(v[19]), "=r"(v[20]),
+        "=r"(v[21]), "=r"(v[22]), "=r"(v[23]), "=r"(v[24]), "=r"(v[25]), "=r"(v[26]), "=r"(v[27]),
+        "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 32; ++i) f[i] = __uint_as_float(v[i]);
+}
+
+__device__ __forceinline__ void pa_st32(uint32_t taddr, const float* f) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
+      "%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),
+      "r"(__float_as_uint(f[0])), "r"(__float_as_uint(f[1])), "r"(__float_as_uint(f[2])),
+      "r"(__float_as_uint(f[3])), "r"(__float_as_uint(f[4])), "r"(__float_as_uint(f[5])),
+      "r"(__float_as_uint(f[6])), "r"(__float_as_uint(f[7])), "r"(__float_as_uint(f[8])),
+      "r"(__float_as_uint(f[9])), "r"(__float_as_uint(f[10])), "r"(__float_as_uint(f[11])),
+      "r"(__float_as_uint(f[12])), "r"(__float_as_uint(f[13])), "r"(__float_as_uint(f[14])),
+      "r"(__float_as_uint(f[15])), "r"(__float_as_uint(f[16])), "r"(__float_as_uint(f[17])),
+      "r"(__float_as_uint(f[18])), "r"(__float_as_uint(f[19])), "r"(__float_as_uint(f[20])),
+      "r"(__float_as_uint(f[21])), "r"(__float_as_uint(f[22])), "r"(__float_as_uint(f[23])),
+      "r"(__float_as_uint(f[24])), "r"(__float_as_uint(f[25])), "r"(__float_as_uint(f[26])),
+      "r"(__float_as_uint(f[27])), "r"(__float_as_uint(f[28])), "r"(__float_as_uint(f[29])),
+      "r"(__float_as_uint(f[30])), "r"(__float_as_uint(f[31]))
+      : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void fence_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+template <int G>
+__global__ void __launch_bounds__(kPaThreads, 1) dmc_prefill_attn_kernel(const PrefillAttnArgs a) {
+  constexpr int D = kPaD;
+  constexpr int ROW = D * 2;          // bytes per bf16 row
+  constexpr int TT = kPaRows / G;     // tokens per tile
+  extern __shared__ __align__(1024) unsigned char smem[];
+  const Layout& L = a.lay;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int tile = blockIdx.x, h = blockIdx.y, s = blockIdx.z;
+  const int bh = (a.first_seq + s) * L.Hkv + h;
+
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kPaMisc);  // [0] S done, [1] O done
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(smem + kPaMisc + 16);
+  int* s_misc = reinterpret_cast<int*>(smem + kPaMisc + 32);       // [0] n_vis max, [1] timeout
+  int* s_len = reinterpret_cast<int*>(smem + kPaMisc + 64);        // [128] slot count after token
+  float* s_om = reinterpret_cast<float*>(smem + kPaMisc + 64 + 512);  // [128] omega
+  unsigned char* s_op = smem + kPaMisc + 64 + 1024;                   // [128] token opens a slot
+
+  const int t0 = a.cu[s], t1 = a.cu[s + 1];
+  if (!(t0 >= 0 && t0 <= t1 && t1 <= a.total_tokens && t1 - t0 <= a.max_seqlen)) return;
+  const int tok0 = t0 + tile * TT;
+  if (tok0 >= t1) return;
+  const int tokN = min(tok0 + TT, t1);
+  const int c = (tok0 - t0) / kPrefillChunk;
+  const int a0 = t0 + c * kPrefillChunk;  // the chunk holding the tile
+  const int cid = (t0 + c * kPrefillChunk) / kPrefillChunk + s;
+  const int base = L.plan[(size_t)h * L.plan_stride + cid];  // slots before the chunk
+  if (base < 0) return;  // the plan failed (capacity or pool); its fault bit is set
+  const int parity = *reinterpret_cast<volatile int*>(&L.ctl[a.layer * 4]);
+  const int len_final = L.lengths[((size_t)a.layer * 2 + parity) * L.NH + bh];
+  const int* ptab = L.page_table + ((size_t)a.layer * L.NH + bh) * L.MPH;
+  const __nv_bfloat16* qg = reinterpret_cast<const __nv_bfloat16*>(a.q);
+
+  // ---- per-token decisions, omega and slot counts of the chunk up to the tile end
+  {
+    const int tau = a0 + tid;
+    int op = 0;
+    float om = 0.f;
+    if (tau < tokN) {
+      op = L.opens[(size_t)tau * L.Hkv + h];
+      float y = 0.f;
+#pragma unroll
+      for (int g = 0; g < G; ++g)
+        y += __bfloat162float(qg[((size_t)tau * L.Hq + (size_t)h * G + g) * D]);
+      om = sigmoidf_(y / (float)G);  // omega = sigmoid(mean of the group's q[0])
+    }
+    s_op[tid] = (unsigned char)op;
+    s_om[tid] = om;
+    // inclusive count of openings up to this token
+    int incl = op;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const int o = __shfl_up_sync(0xffffffffu, incl, off);
+      if (lane >= off) incl += o;
+    }
+    s_len[tid] = incl;  // per-warp prefix for now
+  }
+  if (tid == 0) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(&bars[0])));
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(&bars[1])));
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    s_misc[1] = 0;
+  }
+  if (warp == 0) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_u32(tslot)),
+                 "r"(256));
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+  }
+  __syncthreads();
+  {
+    int add = base;
+    for (int w = 0; w < warp; ++w) add += s_len[w * 32 + 31];
+    __syncthreads();
+    s_len[tid] += add;  // slot count after token a0 + tid
+  }
+  __syncthreads();
+
+  // ---- rows: row r is token tok0 + r / G, query head h * G + r % G
+  const int r = tid;
+  const int tau_r = tok0 + r / G;
+  const bool row_ok = tau_r < tokN;
+  const int nvis = row_ok ? s_len[tau_r - a0] - 1 : 0;  // closed slots this row sees
+  const int nvis_max = s_len[tokN - 1 - a0] - 1;
+  const int vis_hi = min(nvis_max, len_final);          // slots worth loading
+  const int ntiles = (vis_hi + kPaSlots - 1) / kPaSlots;
+
+  const uint32_t sQ = smem_u32(smem + kPaQ);
+  // Q rows (zero rows past the tile's tokens)
+  for (int i = tid; i < kPaRows * 16; i += kPaThreads) {
+    const int rr = i >> 4, j = i & 15;
+    const int tt = tok0 + rr / G;
+    const bool ok = tt < tokN;
+    const char* src = a.q + (((size_t)(ok ? tt : tok0) * L.Hq + (size_t)h * G + rr % G) * ROW) + j * 16;
+    cp_async16_zfill(sQ + pa_swz(rr, j), src, ok);
+  }
+  // K/V rows of slot tile jt into buffer b (zero rows past vis_hi)
+  auto load_kv = [&](int jt, int b) {
+    const uint32_t sK = smem_u32(smem + kPaK + b * kPaTileBytes);
+    const uint32_t sV = smem_u32(smem + kPaV + b * kPaTileBytes);
+    for (int i = tid; i < kPaSlots * 16; i += kPaThreads) {
+      const int rr = i >> 4, j = i & 15;
+      const int slot = jt * kPaSlots + rr;
+      const bool ok = slot < vis_hi;
+      const int page = ok ? ptab[slot / kPage] : 0;
+      const char* src = L.pages + (size_t)page * L.page_bytes + (size_t)(ok ? slot % kPage : 0) * ROW + j * 16;
+      cp_async16_zfill(sK + pa_swz(rr, j), src, ok);
+      cp_async16_zfill(sV + pa_swz(rr, j), src + (size_t)kPage * ROW, ok);
+    }
+  };
+  if (ntiles > 0) load_kv(0, 0);
+  cp_async_commit();
+
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tslot;
+  const uint32_t tS = tmem, tO = tmem + 128;
+  const uint32_t lane_base = (uint32_t)(warp * 32) << 16;  // this warp's TMEM lanes
+  const float qscale = 1.4426950408889634f / sqrtf((float)D);  // log2(e) / sqrt(d_h)
+
+  auto wait_bar = [&](int which, int parity_) {
+    const uint32_t bar = smem_u32(&bars[which]);
+#pragma unroll 1
+    for (int i = 0; i < 64; ++i)
+      if (mbar_try_wait(bar, parity_)) return;
+    const uint64_t tb = globaltimer_ns();
+#pragma unroll 1
+    while (!mbar_try_wait(bar, parity_)) {
+      if (globaltimer_ns() - tb > kWaitLimitNs) {
+        atomicOr(L.error, DMC_FAULT_WAIT_TIMEOUT);
+        s_misc[1] = 1;
+        return;
+      }
+    }
+  };
+
+  float m = -INFINITY, l = 0.f;
+  for (int jt = 0; jt < ntiles; ++jt) {
+    const int b = jt & 1;
+    // P V of the previous tile is done (so are all earlier MMAs): its K/V
+    // buffer and P are free, O holds it
+    if (jt > 0) wait_bar(1, (jt - 1) & 1);
+    if (jt + 1 < ntiles) load_kv(jt + 1, b ^ 1);
+    cp_async_commit();
+    cp_async_wait<1>();  // Q and tile jt have landed (this thread's copies)
+    fence_async_smem();
+    __syncthreads();
+    if (tid == 0) {
+      tc_fence_after();
+      const uint32_t kA = sQ, kB = smem_u32(smem + kPaK + b * kPaTileBytes);
+#pragma unroll
+      for (int kk = 0; kk < D / 16; ++kk) {
+        const uint32_t off = (kk >> 2) * (kPaRows * 128) + (kk & 3) * 32;
+        pa_mma(tS, pa_desc(kA + off, 16, 1024), pa_desc(kB + off, 16, 1024), pa_idesc(false), kk > 0);
+      }
+      pa_commit(smem_u32(&bars[0]));
+    }
+    wait_bar(0, jt & 1);
+    tc_fence_after();
+    // ---- online softmax of this row over the tile's slots
+    const int vis_here = min(max(nvis - jt * kPaSlots, 0), kPaSlots);  // visible columns
+    // TMEM loads are warp-wide: the warp reads as far as its widest row
+    const int vis_warp = __reduce_max_sync(0xffffffffu, vis_here);
+    float mx = -INFINITY;
+    for (int c0 = 0; c0 < vis_warp; c0 += 32) {
+      float f[32];
+      pa_ld32(tS + lane_base + c0, f);
+#pragma unroll
+      for (int i = 0; i < 32; ++i)
+        if (c0 + i < vis_here) mx = fmaxf(mx, f[i] * qscale);
+    }
+    const float mn = fmaxf(m, mx);
+    float sum = 0.f;
+    unsigned char* sP = smem + kPaP;
+    for (int c0 = 0; c0 < kPaSlots; c0 += 32) {
+      float f[32];
+      if (c0 < vis_warp) {
+        pa_ld32(tS + lane_base + c0, f);
+      } else {
+#pragma unroll
+        for (int i = 0; i < 32; ++i) f[i] = 0.f;
+      }
+#pragma unroll
+      for (int i = 0; i < 32; ++i) {
+        const float p = (c0 + i < vis_here) ? exp2f(f[i] * qscale - mn) : 0.f;
+        f[i] = p;
+        sum += p;
+      }
+#pragma unroll
+      for (int q4 = 0; q4 < 4; ++q4) {
+        const uint4 u = Chunk<__nv_bfloat16>::pack(f + q4 * 8);
+        *reinterpret_cast<uint4*>(sP + pa_swz(r, (c0 >> 3) + q4)) = u;
+      }
+    }
+    const float corr = (m == -INFINITY) ? 0.f : exp2f(m - mn);
+    l = l * corr + sum;
+    // rescale O rows whose maximum moved (rows that saw nothing yet hold zeros)
+    const bool resc = jt > 0 && corr != 1.f;
+    if (__any_sync(0xffffffffu, resc)) {
+      const float cr = resc ? corr : 1.f;
+      for (int c0 = 0; c0 < D; c0 += 32) {
+        float f[32];
+        pa_ld32(tO + lane_base + c0, f);
+#pragma unroll
+        for (int i = 0; i < 32; ++i) f[i] *= cr;
+        pa_st32(tO + lane_base + c0, f);
+      }
+      asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+    }
+    if (mn != -INFINITY) m = mn;
+    fence_async_smem();
+    tc_fence_before();
+    __syncthreads();
+    if (tid == 0) {
+      tc_fence_after();
+      const uint32_t pA = smem_u32(smem + kPaP), vB = smem_u32(smem + kPaV + b * kPaTileBytes);
+#pragma unroll
+      for (int kk = 0; kk < kPaSlots / 16; ++kk) {
+        const uint32_t aoff = (kk >> 2) * (kPaRows * 128) + (kk & 3) * 32;
+        pa_mma(tO, pa_desc(pA + aoff, 16, 1024), pa_desc(vB + kk * 2048, kPaRows * 128, 1024),
+               pa_idesc(true), jt > 0 || kk > 0);
+      }
+      pa_commit(smem_u32(&bars[1]));
+    }
+  }
+  if (ntiles > 0) wait_bar(1, (ntiles - 1) & 1);
+  cp_async_wait<0>();
+  tc_fence_after();
+  __syncthreads();  // every thread's reads of the K/V buffers are over
+
+  // ---- the diagonal state of each token: segment sums from the chunk start
+  // raw k, v rows of tokens [a0, tokN) into K buffer 0 / 1 (row-major, 256 B rows)
+  unsigned char* rk = smem + kPaK;
+  unsigned char* rv = smem + kPaK + kPaTileBytes;
+  const int nrows = tokN - a0;
+  for (int i = tid; i < nrows * 16; i += kPaThreads) {
+    const int rr = i >> 4, j = i & 15;
+    const size_t src = ((size_t)(a0 + rr) * L.Hkv + h) * ROW + j * 16;
+    cp_async16(smem_u32(rk + rr * ROW + j * 16), a.k + src);
+    cp_async16(smem_u32(rv + rr * ROW + j * 16), a.v + src);
+  }
+  cp_async_commit();
+  cp_async_wait<0>();
+  __syncthreads();
+  // thread t runs column t of k and of v down the chunk; the running means of
+  // the tile's tokens go to V buffer 0 (keys) and 1 (values) as bf16 rows
+  {
+    const int col = tid;
+    float ak = 0.f, av = 0.f, z = 0.f;
+    if (!s_op[0]) {
+      // the chunk's first token continues a segment: its sums so far
+      const float* cp = a.carry + ((size_t)cid * L.Hkv + h) * (2 * D + 1);
+      ak = cp[col];
+      av = cp[D + col];
+      z = cp[2 * D];
+    }
+    __nv_bfloat16* dk = reinterpret_cast<__nv_bfloat16*>(smem + kPaV);
+    __nv_bfloat16* dv = reinterpret_cast<__nv_bfloat16*>(smem + kPaV + kPaTileBytes);
+    for (int i = 0; i < nrows; ++i) {
+      if (s_op[i]) { ak = 0.f; av = 0.f; z = 0.f; }
+      const float w = s_om[i];
+      const float kx = col == 0 ? 0.f : __bfloat162float(reinterpret_cast<const __nv_bfloat16*>(rk + i * ROW)[col]);
+      const float vx = __bfloat162float(reinterpret_cast<const __nv_bfloat16*>(rv + i * ROW)[col]);
+      ak = fmaf(w, kx, ak);
+      av = fmaf(w, vx, av);
+      z += w;
+      const int ti = a0 + i - tok0;  // row of the tile's token
+      if (ti >= 0) {
+        dk[ti * D + col] = __float2bfloat16_rn(ak / z);
+        dv[ti * D + col] = __float2bfloat16_rn(av / z);
+      }
+    }
+  }
+  __syncthreads();
+
+  // ---- merge the diagonal state and write the row (TMEM loads by every lane)
+  {
+    const int ti = row_ok ? r / G : 0;
+    const __nv_bfloat16* krow = reinterpret_cast<const __nv_bfloat16*>(smem + kPaV) + ti * D;
+    const __nv_bfloat16* vrow = reinterpret_cast<const __nv_bfloat16*>(smem + kPaV + kPaTileBytes) + ti * D;
+    float dsc = 0.f;
+#pragma unroll 4
+    for (int j = 0; j < 16; ++j) {
+      const uint4 qu = *reinterpret_cast<const uint4*>(smem + kPaQ + pa_swz(r, j));
+      const uint4 ku = *reinterpret_cast<const uint4*>(krow + j * 8);
+      float qf[8], kf[8];
+      Chunk<__nv_bfloat16>::unpack(qu, qf);
+      Chunk<__nv_bfloat16>::unpack(ku, kf);
+#pragma unroll
+      for (int e = 0; e < 8; ++e) dsc = fmaf(qf[e], kf[e], dsc);
+    }
+    dsc *= qscale;  // k~[0] = 0, so q[0] drops out
+    const float M = fmaxf(m, dsc);
+    const float cO = (m == -INFINITY) ? 0.f : exp2f(m - M);
+    const float cD = exp2f(dsc - M);
+    const float inv = 1.f / (l * cO + cD);
+    char* orow = a.out + ((size_t)(row_ok ? tau_r : tok0) * L.Hq + (size_t)h * G + r % G) * ROW;
+    for (int c0 = 0; c0 < D; c0 += 32) {
+      float f[32];
+      if (ntiles > 0) pa_ld32(tO + lane_base + c0, f);  // CTA-uniform
+      if (ntiles == 0 || m == -INFINITY) {
+#pragma unroll
+        for (int i = 0; i < 32; ++i) f[i] = 0.f;
+      }
+      if (row_ok) {
+#pragma unroll
+        for (int q4 = 0; q4 < 4; ++q4) {
+          float vf[8], o[8];
+          Chunk<__nv_bfloat16>::unpack(*reinterpret_cast<const uint4*>(vrow + c0 + q4 * 8), vf);
+#pragma unroll
+          for (int e = 0; e < 8; ++e) o[e] = (f[q4 * 8 + e] * cO + vf[e] * cD) * inv;
+          *reinterpret_cast<uint4*>(orow + (c0 + q4 * 8) * 2) = Chunk<__nv_bfloat16>::pack(o);
+        }
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(256));
+  }
+}
+
+bool prefill_attn_supported(const Layout& L) {
+  return L.esize == 2 && L.D == kPaD && (L.G == 1 || L.G == 2 || L.G == 4 || L.G == 8);
+}
+
+template <int G>
+static cudaError_t launch_pa(const PrefillAttnArgs& a, cudaStream_t stream) {
+  cudaError_t e = cudaFuncSetAttribute(dmc_prefill_attn_kernel<G>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, kPaSmem);
+  if (e != cudaSuccess) return e;
+  constexpr int TT = kPaRows / G;
+  const int tiles = (a.max_seqlen + TT - 1) / TT;
+  if (tiles == 0) return cudaSuccess;
+  dmc_prefill_attn_kernel<G><<<dim3(tiles, a.lay.Hkv, a.num_seqs), kPaThreads, kPaSmem, stream>>>(a);
+  return cudaGetLastError();
+}
+
+cudaError_t prefill_attn_launch(const Layout& L, int layer, int first_seq, int num_seqs,
+                                const void* q, const void* k, const void* v, const int* cu,
+                                int total_tokens, int max_seqlen, const float* carry, void* out,
+                                cudaStream_t stream) {
+  PrefillAttnArgs a;
+  a.lay = L;
+  a.layer = layer;
+  a.first_seq = first_seq;
+  a.num_seqs = num_seqs;
+  a.q = static_cast<const char*>(q);
+  a.k = static_cast<const char*>(k);
+  a.v = static_cast<const char*>(v);
+  a.cu = cu;
+  a.total_tokens = total_tokens;
+  a.max_seqlen = max_seqlen;
+  a.carry = carry;
+  a.out = static_cast<char*>(out);
+  switch (L.G) {
+    case 1: return launch_pa<1>(a, stream);
+    case 2: return launch_pa<2>(a, stream);
+    case 4: return launch_pa<4>(a, stream);
+    case 8: return launch_pa<8>(a, stream);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+}  // namespace dmc

@@ -146,13 +146,15 @@ def _draw_tokens(n, wl: Workload, p_layer, g, device, want_full_q: bool):
     return q, k, v
 
 
-def gen_prompt(wl: Workload, layer: int, device, seqs=None, p=None):
+def gen_prompt(wl: Workload, layer: int, device, seqs=None, p=None, full_q: bool = False):
     """Prompt inputs of one layer for the sequences `seqs` (default: all).
 
     Returns dict q0 [sum T, Hq] (first neuron of every query), k, v
     [sum T, Hkv, d] in the workload dtype, cu_seqlens int32 [n+1] (on `device`)
     and the per-sequence lengths (numpy). Each sequence has its own generator
-    stream, so any subset is reproducible."""
+    stream, so any subset is reproducible. With full_q the whole queries are
+    drawn too ("q" [sum T, Hq, d], q0 = its first neuron); that draws more
+    numbers, so those prompts differ from the default ones."""
     if seqs is None:
         seqs = range(wl.batch)
     seqs = list(seqs)
@@ -163,20 +165,25 @@ def gen_prompt(wl: Workload, layer: int, device, seqs=None, p=None):
     H, Hq, d = wl.num_kv_heads, wl.num_q_heads, wl.head_dim
     dt = wl.torch_dtype
     q0 = torch.empty((total, Hq), dtype=dt, device=device)
+    qf = torch.empty((total, Hq, d), dtype=dt, device=device) if full_q else None
     k = torch.empty((total, H, d), dtype=dt, device=device)
     v = torch.empty((total, H, d), dtype=dt, device=device)
     off = 0
     for b, n in zip(seqs, lens):
         n = int(n)
         g = _gen(device, derive_seed(wl.seed, 1, layer, b))
-        qb, kb, vb = _draw_tokens(n, wl, p[layer], g, device, want_full_q=False)
-        q0[off:off + n] = qb.to(dt)
+        qb, kb, vb = _draw_tokens(n, wl, p[layer], g, device, want_full_q=full_q)
+        if full_q:
+            qf[off:off + n] = qb.to(dt)
+            q0[off:off + n] = qb[:, :, 0].to(dt)
+        else:
+            q0[off:off + n] = qb.to(dt)
         k[off:off + n] = kb.to(dt)
         v[off:off + n] = vb.to(dt)
         off += n
     cu = np.zeros(len(seqs) + 1, dtype=np.int32)
     cu[1:] = np.cumsum(lens)
-    return {"q0": q0, "k": k, "v": v,
+    return {"q0": q0, "q": qf, "k": k, "v": v,
             "cu_seqlens": torch.as_tensor(cu, device=device),
             "lens": lens, "max_seqlen": int(lens.max()) if len(lens) else 0}
 

@@ -69,6 +69,7 @@ def test_create_rejects_bad_arena_on_the_host(lib):
 def test_null_handle_is_rejected(lib):
     assert P.dmc_decode_step(None, 0, 16, 16, 16, 16, 0) == P.DMC_ERR_INVALID_ARG
     assert P.dmc_cache_lengths(None, 0, 16, 0) == P.DMC_ERR_INVALID_ARG
+    assert P.dmc_prefill_attention(None, 0, 0, 1, 16, 16, 16, 16, 1, 1, 16, 0) == P.DMC_ERR_INVALID_ARG
     assert P.dmc_cache_destroy(None) == P.DMC_OK
 
 

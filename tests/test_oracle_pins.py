@@ -260,6 +260,30 @@ def test_sequential_equals_training_mask(seed):
     assert np.allclose(r["out"], R.masked_attention(k, v, q), atol=1e-12)
 
 
+@pytest.mark.parametrize("seed", [3, 4])
+def test_prompt_attention_equals_training_mask(seed):
+    """Prompt outputs token by token (inference) = the masked attention over all
+    unrolled states (training formulation), for a group of 2 queries."""
+    rng = np.random.default_rng(seed)
+    n, d = 23, 6
+    k, v = rng.normal(size=(n, d)), rng.normal(size=(n, d))
+    q = rng.normal(size=(n, 2, d))
+    assert np.allclose(R.prompt_attention(k, v, q), R.masked_attention(k, v, q), atol=1e-12)
+
+
+def test_prompt_attention_all_accumulate_is_running_mean():
+    """k[0] >= 0 everywhere: one segment, every token sees only the running
+    omega-weighted mean of the values so far."""
+    rng = np.random.default_rng(5)
+    n, d = 17, 5
+    k, v = rng.normal(size=(n, d)), rng.normal(size=(n, d))
+    k[:, 0] = np.abs(k[:, 0]) + 0.1
+    q = rng.normal(size=(n, 1, d))
+    w = 1.0 / (1.0 + np.exp(-q[:, 0, 0]))
+    want = np.cumsum(w[:, None] * v, axis=0) / np.cumsum(w)[:, None]
+    assert np.allclose(R.prompt_attention(k, v, q)[:, 0], want, atol=1e-12)
+
+
 def test_gqa_equal_group_q0_reduces_to_mha_omega():
     rng = _rng(11)
     n, d, G = 20, 6, 4
