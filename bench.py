@@ -57,6 +57,8 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--pa-layers", type=int, default=4,
+                    help="layers of the prompt-attention measurement (0 skips it)")
     ap.add_argument("--graph", action="store_true",
                     help="replay the step's launches from CUDA graphs instead of launching from the host")
     return ap.parse_args()
@@ -435,11 +437,99 @@ def run_ours(args, rank, world, dist):
     }
 
     # ---- end to end: same step through the C ABI with pinned host buffers
+    if args.pa_layers > 0:
+        res["prompt_attention"] = run_prompt_attention(args, wl, dev, stream, dist)
     if not args.no_e2e:
         res["e2e"] = run_e2e(args, wl, cache, prompts, qd, kd, vd, outs, steps_dec, dev, stream, L_,
                              barrier, dist, world, local)
     del qd, kd, vd
     return res
+
+
+def run_prompt_attention(args, wl, dev, stream, dist):
+    """Prompt-phase attention (dmc_prefill_attention) on the workload's prompt
+    shape, over `--pa-layers` layers with full queries: per pass, reset then
+    one call per layer. The tensor-core kernel's time is the call's time minus
+    that of dmc_prefill_compress on the same prompts (the call runs the same
+    compression first). Algorithmic FLOPs: 4 * head_dim per (query row,
+    visible slot) plus the diagonal state, the useful part of S = Q K^T and
+    O = P V."""
+    import torch
+    import paper_2403_09636_gb300 as P
+    from paper_2403_09636_gb300 import synthetic as S
+
+    G, D = wl.group, wl.head_dim
+    if not (wl.dtype == "bf16" and D == 128 and G in (1, 2, 4, 8)):
+        return {"skipped": "prompt attention runs on bf16 caches with head_dim 128 and groups 1/2/4/8"}
+    Lp = max(1, min(args.pa_layers, wl.num_layers))
+    p = S.append_prob(wl)
+    prompts = [S.gen_prompt(wl, l, dev, p=p, full_q=True) for l in range(Lp)]
+    outs = [torch.empty_like(pr["q"]) for pr in prompts]
+    flops = 0
+    pages = 0
+    for pr in prompts:
+        cu = pr["cu_seqlens"].to(torch.int64)
+        opens = (pr["k"][:, :, 0] < 0).to(torch.int64)
+        opens[cu[:-1]] = 1                                     # first token of an empty head
+        seg = torch.cumsum(opens, 0)                           # slots after each token (global)
+        before = torch.cat([torch.zeros_like(seg[:1]), seg])[cu[:-1]]
+        nseq = torch.repeat_interleave(torch.arange(cu.numel() - 1, device=dev), cu[1:] - cu[:-1])
+        len_after = seg - before[nseq]                         # per (token, KV head)
+        flops += int(((len_after - 1).sum() * 4 * D + len_after.numel() * 4 * D) * G)
+        pages += int(((len_after[cu[1:] - 1] + 31) // 32).sum())
+    lens = S.prompt_lengths(wl)
+    cache = P.DmcCache(Lp, wl.batch, wl.num_q_heads, wl.num_kv_heads, D, wl.torch_dtype,
+                       int(lens.max()) + 2, pages + 64, int(lens.sum()), device=dev)
+    h, sh = cache.handle, stream.cuda_stream
+
+    def attn_pass():
+        cache.reset(stream)
+        for l, (pr, o) in enumerate(zip(prompts, outs)):
+            cache.prefill_attention(l, pr["q"], pr["k"], pr["v"], pr["cu_seqlens"], pr["max_seqlen"],
+                                    o, stream=stream)
+
+    def compress_pass():
+        cache.reset(stream)
+        for l, pr in enumerate(prompts):
+            cache.prefill(l, pr["q0"], pr["k"], pr["v"], pr["cu_seqlens"], pr["max_seqlen"],
+                          stream=stream)
+
+    def timed(fn, reps):
+        for _ in range(2):
+            fn()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(reps):
+            fn()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) / reps
+
+    reps = max(3, args.steps)
+    ms_attn = timed(attn_pass, reps)
+    ms_comp = timed(compress_pass, reps)
+    st, bits, _ = cache.status()
+    if st != 0:
+        raise RuntimeError(f"device fault in prompt attention: status {st} bits {bits:#x}")
+    ms_attn, ms_comp = max_over_ranks(dist, [ms_attn, ms_comp], dev)
+    tokens = sum(int(pr["cu_seqlens"][-1]) for pr in prompts)
+    kern_ms = max(ms_attn - ms_comp, 1e-6)
+    tflops = flops / (kern_ms / 1e3) / 1e12
+    peak = 1900.0
+    try:
+        peak = float(json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))["bf16_tflops"])
+        peak_kind = "measured dense bf16 (cuBLAS burst)"
+    except Exception:
+        peak_kind = "fallback dense bf16"
+    return {"layers": Lp, "prompt_tokens_per_layer": tokens // Lp,
+            "tokens_per_s": tokens / (ms_attn / 1e3),
+            "ms_per_layer_with_compress": ms_attn / Lp, "ms_per_layer_compress_only": ms_comp / Lp,
+            "roofline": {"kernel": f"dmc_prefill_attn_kernel<{G}>", "bound": "tensor",
+                         "achieved": tflops, "peak": peak, "peak_kind": peak_kind,
+                         "unit": "TFLOP/s", "frac": tflops / peak,
+                         "algorithmic_flops_per_layer": flops / Lp,
+                         "timing": "call time minus dmc_prefill_compress time on the same prompts"}}
 
 
 def run_e2e(args, wl, cache, prompts, qd, kd, vd, outs, steps_dec, dev, stream, L_, barrier, dist,

@@ -9,14 +9,16 @@
 // query i therefore sees the final values of slots [0, len(i) - 1) and one
 // "diagonal" state.
 //
-// One CTA of 4 warps per (128 query rows, KV head, sequence); a row is a
+// One CTA of 8 warps per (128 query rows, KV head, sequence); a row is a
 // (token, query head of the group) pair, token-major, so a group of G queries
 // shares every K/V tile. The closed slots are read from the cache pages that
 // the prefill scan has just written, in tiles of 128 slots:
 //   S = Q K^T          tcgen05.mma kind::f16, M = N = 128, K = head_dim, into TMEM
-//   softmax            one thread per row: tcgen05.ld of its S row, the
-//                      staircase mask (slot < len(i) - 1), online softmax in
-//                      the log2 domain, P rounded to bf16 into shared memory
+//   softmax            two threads per row, each half of its columns:
+//                      tcgen05.ld of S, the staircase mask (slot < len(i) - 1),
+//                      online softmax in the log2 domain (the halves trade
+//                      their maxima through shared memory), P rounded to bf16
+//                      into shared memory
 //   O += P V           tcgen05.mma with V as an MN-major B operand, into TMEM
 // The diagonal state of each token is rebuilt at the end from the prompt's
 // k, v rows of the token's 128-token chunk and the segment sums the prefill
@@ -29,13 +31,13 @@ namespace dmc {
 
 constexpr int kPaRows = 128;     // query rows per tile (M)
 constexpr int kPaSlots = 128;    // slots per K/V tile (N of S, K of P V)
-constexpr int kPaThreads = 128;  // one thread per query row
+constexpr int kPaThreads = 256;  // two threads per query row, each half of its columns
 constexpr int kPaD = 128;        // head_dim handled by this kernel
 constexpr int kPaTileBytes = kPaRows * kPaD * 2;  // 32 KB: [128 rows][256 B]
-// dynamic shared memory: Q | K0 | K1 | V0 | V1 | P | misc
-constexpr int kPaQ = 0, kPaK = kPaTileBytes, kPaV = 3 * kPaTileBytes, kPaP = 5 * kPaTileBytes;
-constexpr int kPaMisc = 6 * kPaTileBytes;
-constexpr int kPaSmem = kPaMisc + 2048;
+// dynamic shared memory: Q | K (then P) | V | misc, 100 KB: two CTAs per SM
+constexpr int kPaQ = 0, kPaK = kPaTileBytes, kPaV = 2 * kPaTileBytes, kPaP = kPaK;
+constexpr int kPaMisc = 3 * kPaTileBytes;
+constexpr int kPaSmem = kPaMisc + 4096;
 
 struct PrefillAttnArgs {
   Layout lay;
@@ -129,10 +131,11 @@ __device__ __forceinline__ void fence_async_smem() {
 }
 
 template <int G>
-__global__ void __launch_bounds__(kPaThreads, 1) dmc_prefill_attn_kernel(const PrefillAttnArgs a) {
+__global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const PrefillAttnArgs a) {
   constexpr int D = kPaD;
   constexpr int ROW = D * 2;          // bytes per bf16 row
   constexpr int TT = kPaRows / G;     // tokens per tile
+  constexpr int HALF = kPaSlots / 2;  // columns of S (and of O) per thread
   extern __shared__ __align__(1024) unsigned char smem[];
   const Layout& L = a.lay;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -141,10 +144,12 @@ __global__ void __launch_bounds__(kPaThreads, 1) dmc_prefill_attn_kernel(const P
 
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kPaMisc);  // [0] S done, [1] O done
   uint32_t* tslot = reinterpret_cast<uint32_t*>(smem + kPaMisc + 16);
-  int* s_misc = reinterpret_cast<int*>(smem + kPaMisc + 32);       // [0] n_vis max, [1] timeout
-  int* s_len = reinterpret_cast<int*>(smem + kPaMisc + 64);        // [128] slot count after token
-  float* s_om = reinterpret_cast<float*>(smem + kPaMisc + 64 + 512);  // [128] omega
-  unsigned char* s_op = smem + kPaMisc + 64 + 1024;                   // [128] token opens a slot
+  int* s_len = reinterpret_cast<int*>(smem + kPaMisc + 64);            // [128] slots after token
+  float* s_om = reinterpret_cast<float*>(smem + kPaMisc + 64 + 512);   // [128] omega
+  float* s_rz = reinterpret_cast<float*>(smem + kPaMisc + 64 + 1024);  // [128] 1 / z after token
+  float* s_x = reinterpret_cast<float*>(smem + kPaMisc + 64 + 1536);   // [2][128] row exchange
+  float* s_y = reinterpret_cast<float*>(smem + kPaMisc + 64 + 2560);   // [2][128] row exchange
+  unsigned char* s_op = smem + kPaMisc + 64 + 3584;                    // [128] token opens a slot
 
   const int t0 = a.cu[s], t1 = a.cu[s + 1];
   if (!(t0 >= 0 && t0 <= t1 && t1 <= a.total_tokens && t1 - t0 <= a.max_seqlen)) return;
@@ -160,9 +165,10 @@ __global__ void __launch_bounds__(kPaThreads, 1) dmc_prefill_attn_kernel(const P
   const int len_final = L.lengths[((size_t)a.layer * 2 + parity) * L.NH + bh];
   const int* ptab = L.page_table + ((size_t)a.layer * L.NH + bh) * L.MPH;
   const __nv_bfloat16* qg = reinterpret_cast<const __nv_bfloat16*>(a.q);
+  const float* carry = a.carry + ((size_t)cid * L.Hkv + h) * (2 * D + 1);
 
   // ---- per-token decisions, omega and slot counts of the chunk up to the tile end
-  {
+  if (tid < kPrefillChunk) {
     const int tau = a0 + tid;
     int op = 0;
     float om = 0.f;
@@ -176,20 +182,18 @@ __global__ void __launch_bounds__(kPaThreads, 1) dmc_prefill_attn_kernel(const P
     }
     s_op[tid] = (unsigned char)op;
     s_om[tid] = om;
-    // inclusive count of openings up to this token
-    int incl = op;
+    int incl = op;  // openings up to this token, within the warp for now
 #pragma unroll
     for (int off = 1; off < 32; off <<= 1) {
       const int o = __shfl_up_sync(0xffffffffu, incl, off);
       if (lane >= off) incl += o;
     }
-    s_len[tid] = incl;  // per-warp prefix for now
+    s_len[tid] = incl;
   }
   if (tid == 0) {
     asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(&bars[0])));
     asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(&bars[1])));
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-    s_misc[1] = 0;
   }
   if (warp == 0) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
@@ -198,16 +202,29 @@ __global__ void __launch_bounds__(kPaThreads, 1) dmc_prefill_attn_kernel(const P
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
   }
   __syncthreads();
-  {
-    int add = base;
+  int add = base;
+  if (tid < kPrefillChunk)
     for (int w = 0; w < warp; ++w) add += s_len[w * 32 + 31];
-    __syncthreads();
-    s_len[tid] += add;  // slot count after token a0 + tid
+  if (warp == 4) {
+    // 1 / z of every token of the chunk (the same for all columns): the
+    // segment's summed omega, continuing the carried sums at the chunk start
+    if (lane == 0) {
+      float z = s_op[0] ? 0.f : carry[2 * D];
+      const int n = tokN - a0;
+      for (int i = 0; i < n; ++i) {
+        if (s_op[i]) z = 0.f;
+        z += s_om[i];
+        s_rz[i] = 1.f / z;
+      }
+    }
   }
   __syncthreads();
+  if (tid < kPrefillChunk) s_len[tid] += add;  // slot count after token a0 + tid
+  __syncthreads();
 
-  // ---- rows: row r is token tok0 + r / G, query head h * G + r % G
-  const int r = tid;
+  // ---- thread (r, hf): query row r (token tok0 + r / G, query head h G + r % G),
+  // columns [hf * 64, hf * 64 + 64) of its S and O rows
+  const int r = tid & (kPaRows - 1), hf = tid >> 7;
   const int tau_r = tok0 + r / G;
   const bool row_ok = tau_r < tokN;
   const int nvis = row_ok ? s_len[tau_r - a0] - 1 : 0;  // closed slots this row sees
@@ -216,7 +233,6 @@ __global__ void __launch_bounds__(kPaThreads, 1) dmc_prefill_attn_kernel(const P
   const int ntiles = (vis_hi + kPaSlots - 1) / kPaSlots;
 
   const uint32_t sQ = smem_u32(smem + kPaQ);
-  // Q rows (zero rows past the tile's tokens)
   for (int i = tid; i < kPaRows * 16; i += kPaThreads) {
     const int rr = i >> 4, j = i & 15;
     const int tt = tok0 + rr / G;
@@ -224,10 +240,9 @@ __global__ void __launch_bounds__(kPaThreads, 1) dmc_prefill_attn_kernel(const P
     const char* src = a.q + (((size_t)(ok ? tt : tok0) * L.Hq + (size_t)h * G + rr % G) * ROW) + j * 16;
     cp_async16_zfill(sQ + pa_swz(rr, j), src, ok);
   }
-  // K/V rows of slot tile jt into buffer b (zero rows past vis_hi)
-  auto load_kv = [&](int jt, int b) {
-    const uint32_t sK = smem_u32(smem + kPaK + b * kPaTileBytes);
-    const uint32_t sV = smem_u32(smem + kPaV + b * kPaTileBytes);
+  auto load_kv = [&](int jt) {
+    const uint32_t sK = smem_u32(smem + kPaK);
+    const uint32_t sV = smem_u32(smem + kPaV);
     for (int i = tid; i < kPaSlots * 16; i += kPaThreads) {
       const int rr = i >> 4, j = i & 15;
       const int slot = jt * kPaSlots + rr;
@@ -238,7 +253,7 @@ __global__ void __launch_bounds__(kPaThreads, 1) dmc_prefill_attn_kernel(const P
       cp_async16_zfill(sV + pa_swz(rr, j), src + (size_t)kPage * ROW, ok);
     }
   };
-  if (ntiles > 0) load_kv(0, 0);
+  if (ntiles > 0) load_kv(0);
   cp_async_commit();
 
   tc_fence_before();
@@ -246,39 +261,33 @@ __global__ void __launch_bounds__(kPaThreads, 1) dmc_prefill_attn_kernel(const P
   tc_fence_after();
   const uint32_t tmem = *tslot;
   const uint32_t tS = tmem, tO = tmem + 128;
-  const uint32_t lane_base = (uint32_t)(warp * 32) << 16;  // this warp's TMEM lanes
-  const float qscale = 1.4426950408889634f / sqrtf((float)D);  // log2(e) / sqrt(d_h)
+  const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;  // this warp's TMEM lanes
+  const uint32_t col0 = hf * HALF;                                // this thread's first column
+  const float qscale = 1.4426950408889634f / sqrtf((float)D);   // log2(e) / sqrt(d_h)
 
-  auto wait_bar = [&](int which, int parity_) {
+  auto wait_bar = [&](int which, int ph) {
     const uint32_t bar = smem_u32(&bars[which]);
 #pragma unroll 1
     for (int i = 0; i < 64; ++i)
-      if (mbar_try_wait(bar, parity_)) return;
+      if (mbar_try_wait(bar, ph)) return;
     const uint64_t tb = globaltimer_ns();
 #pragma unroll 1
-    while (!mbar_try_wait(bar, parity_)) {
+    while (!mbar_try_wait(bar, ph)) {
       if (globaltimer_ns() - tb > kWaitLimitNs) {
         atomicOr(L.error, DMC_FAULT_WAIT_TIMEOUT);
-        s_misc[1] = 1;
         return;
       }
     }
   };
 
-  float m = -INFINITY, l = 0.f;
+  float m = -INFINITY, l = 0.f;  // l: this thread's half of the row sum
   for (int jt = 0; jt < ntiles; ++jt) {
-    const int b = jt & 1;
-    // P V of the previous tile is done (so are all earlier MMAs): its K/V
-    // buffer and P are free, O holds it
-    if (jt > 0) wait_bar(1, (jt - 1) & 1);
-    if (jt + 1 < ntiles) load_kv(jt + 1, b ^ 1);
-    cp_async_commit();
-    cp_async_wait<1>();  // Q and tile jt have landed (this thread's copies)
+    cp_async_wait<0>();  // Q and tile jt have landed (this thread's copies)
     fence_async_smem();
     __syncthreads();
     if (tid == 0) {
       tc_fence_after();
-      const uint32_t kA = sQ, kB = smem_u32(smem + kPaK + b * kPaTileBytes);
+      const uint32_t kA = sQ, kB = smem_u32(smem + kPaK);
 #pragma unroll
       for (int kk = 0; kk < D / 16; ++kk) {
         const uint32_t off = (kk >> 2) * (kPaRows * 128) + (kk & 3) * 32;
@@ -286,55 +295,57 @@ __global__ void __launch_bounds__(kPaThreads, 1) dmc_prefill_attn_kernel(const P
       }
       pa_commit(smem_u32(&bars[0]));
     }
-    wait_bar(0, jt & 1);
+    wait_bar(0, jt & 1);  // S is in TMEM; the K buffer is free for P
     tc_fence_after();
-    // ---- online softmax of this row over the tile's slots
-    const int vis_here = min(max(nvis - jt * kPaSlots, 0), kPaSlots);  // visible columns
-    // TMEM loads are warp-wide: the warp reads as far as its widest row
-    const int vis_warp = __reduce_max_sync(0xffffffffu, vis_here);
+    // ---- online softmax: this thread's half of the row
+    const int vis_row = min(max(nvis - jt * kPaSlots, 0), kPaSlots);  // visible columns of the row
+    const int vis_me = min(max(vis_row - (int)col0, 0), HALF);         // ... in this half
+    const int vis_warp = __reduce_max_sync(0xffffffffu, vis_me);       // TMEM loads are warp-wide
     float mx = -INFINITY;
     for (int c0 = 0; c0 < vis_warp; c0 += 32) {
       float f[32];
-      pa_ld32(tS + lane_base + c0, f);
+      pa_ld32(tS + lane_base + col0 + c0, f);
 #pragma unroll
       for (int i = 0; i < 32; ++i)
-        if (c0 + i < vis_here) mx = fmaxf(mx, f[i] * qscale);
+        if (c0 + i < vis_me) mx = fmaxf(mx, f[i] * qscale);
     }
-    const float mn = fmaxf(m, mx);
+    s_x[hf * kPaRows + r] = mx;
+    __syncthreads();
+    const float mn = fmaxf(m, fmaxf(mx, s_x[(hf ^ 1) * kPaRows + r]));
     float sum = 0.f;
     unsigned char* sP = smem + kPaP;
-    for (int c0 = 0; c0 < kPaSlots; c0 += 32) {
+    for (int c0 = 0; c0 < HALF; c0 += 32) {
       float f[32];
       if (c0 < vis_warp) {
-        pa_ld32(tS + lane_base + c0, f);
+        pa_ld32(tS + lane_base + col0 + c0, f);
       } else {
 #pragma unroll
         for (int i = 0; i < 32; ++i) f[i] = 0.f;
       }
 #pragma unroll
       for (int i = 0; i < 32; ++i) {
-        const float p = (c0 + i < vis_here) ? exp2f(f[i] * qscale - mn) : 0.f;
+        const float p = (c0 + i < vis_me) ? exp2f(f[i] * qscale - mn) : 0.f;
         f[i] = p;
         sum += p;
       }
 #pragma unroll
-      for (int q4 = 0; q4 < 4; ++q4) {
-        const uint4 u = Chunk<__nv_bfloat16>::pack(f + q4 * 8);
-        *reinterpret_cast<uint4*>(sP + pa_swz(r, (c0 >> 3) + q4)) = u;
-      }
+      for (int q4 = 0; q4 < 4; ++q4)
+        *reinterpret_cast<uint4*>(sP + pa_swz(r, ((col0 + c0) >> 3) + q4)) =
+            Chunk<__nv_bfloat16>::pack(f + q4 * 8);
     }
     const float corr = (m == -INFINITY) ? 0.f : exp2f(m - mn);
     l = l * corr + sum;
-    // rescale O rows whose maximum moved (rows that saw nothing yet hold zeros)
+    // rescale this half of O rows whose maximum moved (rows that saw nothing
+    // yet hold zeros)
     const bool resc = jt > 0 && corr != 1.f;
     if (__any_sync(0xffffffffu, resc)) {
       const float cr = resc ? corr : 1.f;
-      for (int c0 = 0; c0 < D; c0 += 32) {
+      for (int c0 = 0; c0 < HALF; c0 += 32) {
         float f[32];
-        pa_ld32(tO + lane_base + c0, f);
+        pa_ld32(tO + lane_base + col0 + c0, f);
 #pragma unroll
         for (int i = 0; i < 32; ++i) f[i] *= cr;
-        pa_st32(tO + lane_base + c0, f);
+        pa_st32(tO + lane_base + col0 + c0, f);
       }
       asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
     }
@@ -344,7 +355,7 @@ __global__ void __launch_bounds__(kPaThreads, 1) dmc_prefill_attn_kernel(const P
     __syncthreads();
     if (tid == 0) {
       tc_fence_after();
-      const uint32_t pA = smem_u32(smem + kPaP), vB = smem_u32(smem + kPaV + b * kPaTileBytes);
+      const uint32_t pA = smem_u32(smem + kPaP), vB = smem_u32(smem + kPaV);
 #pragma unroll
       for (int kk = 0; kk < kPaSlots / 16; ++kk) {
         const uint32_t aoff = (kk >> 2) * (kPaRows * 128) + (kk & 3) * 32;
@@ -353,95 +364,91 @@ __global__ void __launch_bounds__(kPaThreads, 1) dmc_prefill_attn_kernel(const P
       }
       pa_commit(smem_u32(&bars[1]));
     }
+    // P V done: O holds this tile, the K (P) and V buffers are free
+    wait_bar(1, jt & 1);
+    if (jt + 1 < ntiles) load_kv(jt + 1);
+    cp_async_commit();
   }
-  if (ntiles > 0) wait_bar(1, (ntiles - 1) & 1);
   cp_async_wait<0>();
   tc_fence_after();
   __syncthreads();  // every thread's reads of the K/V buffers are over
 
   // ---- the diagonal state of each token: segment sums from the chunk start
-  // raw k, v rows of tokens [a0, tokN) into K buffer 0 / 1 (row-major, 256 B rows)
+  // Raw k, v rows of tokens [a0, tokN) go to the K / V buffers as 256-byte rows
+  // whose 16-byte chunks are XOR-swizzled by row (conflict-free row reads
+  // below); the running means then replace them in place.
+  auto scr = [&](int i, int col) { return i * ROW + ((((col >> 3) ^ (i & 15))) << 4) + (col & 7) * 2; };
   unsigned char* rk = smem + kPaK;
-  unsigned char* rv = smem + kPaK + kPaTileBytes;
+  unsigned char* rv = smem + kPaV;
   const int nrows = tokN - a0;
   for (int i = tid; i < nrows * 16; i += kPaThreads) {
     const int rr = i >> 4, j = i & 15;
     const size_t src = ((size_t)(a0 + rr) * L.Hkv + h) * ROW + j * 16;
-    cp_async16(smem_u32(rk + rr * ROW + j * 16), a.k + src);
-    cp_async16(smem_u32(rv + rr * ROW + j * 16), a.v + src);
+    cp_async16(smem_u32(rk + scr(rr, j * 8)), a.k + src);
+    cp_async16(smem_u32(rv + scr(rr, j * 8)), a.v + src);
   }
   cp_async_commit();
   cp_async_wait<0>();
   __syncthreads();
-  // thread t runs column t of k and of v down the chunk; the running means of
-  // the tile's tokens go to V buffer 0 (keys) and 1 (values) as bf16 rows
+  // thread t runs column t % 128 of k (t < 128) or of v down the chunk
   {
-    const int col = tid;
-    float ak = 0.f, av = 0.f, z = 0.f;
-    if (!s_op[0]) {
-      // the chunk's first token continues a segment: its sums so far
-      const float* cp = a.carry + ((size_t)cid * L.Hkv + h) * (2 * D + 1);
-      ak = cp[col];
-      av = cp[D + col];
-      z = cp[2 * D];
-    }
-    __nv_bfloat16* dk = reinterpret_cast<__nv_bfloat16*>(smem + kPaV);
-    __nv_bfloat16* dv = reinterpret_cast<__nv_bfloat16*>(smem + kPaV + kPaTileBytes);
+    const int col = tid & (D - 1);
+    const bool isv = tid >= D;
+    unsigned char* buf = isv ? rv : rk;
+    float acc = s_op[0] ? 0.f : carry[(isv ? D : 0) + col];
     for (int i = 0; i < nrows; ++i) {
-      if (s_op[i]) { ak = 0.f; av = 0.f; z = 0.f; }
-      const float w = s_om[i];
-      const float kx = col == 0 ? 0.f : __bfloat162float(reinterpret_cast<const __nv_bfloat16*>(rk + i * ROW)[col]);
-      const float vx = __bfloat162float(reinterpret_cast<const __nv_bfloat16*>(rv + i * ROW)[col]);
-      ak = fmaf(w, kx, ak);
-      av = fmaf(w, vx, av);
-      z += w;
-      const int ti = a0 + i - tok0;  // row of the tile's token
-      if (ti >= 0) {
-        dk[ti * D + col] = __float2bfloat16_rn(ak / z);
-        dv[ti * D + col] = __float2bfloat16_rn(av / z);
-      }
+      if (s_op[i]) acc = 0.f;
+      __nv_bfloat16* e = reinterpret_cast<__nv_bfloat16*>(buf + scr(i, col));
+      float x = __bfloat162float(*e);
+      if (!isv && col == 0) x = 0.f;  // k[0] <- 0 (Algorithm 1)
+      acc = fmaf(s_om[i], x, acc);
+      *e = __float2bfloat16_rn(acc * s_rz[i]);  // this token's running mean
     }
   }
   __syncthreads();
 
   // ---- merge the diagonal state and write the row (TMEM loads by every lane)
-  {
-    const int ti = row_ok ? r / G : 0;
-    const __nv_bfloat16* krow = reinterpret_cast<const __nv_bfloat16*>(smem + kPaV) + ti * D;
-    const __nv_bfloat16* vrow = reinterpret_cast<const __nv_bfloat16*>(smem + kPaV + kPaTileBytes) + ti * D;
-    float dsc = 0.f;
-#pragma unroll 4
-    for (int j = 0; j < 16; ++j) {
-      const uint4 qu = *reinterpret_cast<const uint4*>(smem + kPaQ + pa_swz(r, j));
-      const uint4 ku = *reinterpret_cast<const uint4*>(krow + j * 8);
-      float qf[8], kf[8];
-      Chunk<__nv_bfloat16>::unpack(qu, qf);
-      Chunk<__nv_bfloat16>::unpack(ku, kf);
+  const int ti = (row_ok ? r / G : 0) + (tok0 - a0);  // the token's row in the staged chunk
+  const unsigned char* kt = rk;
+  const unsigned char* vt = rv;
+  float dp = 0.f;
 #pragma unroll
-      for (int e = 0; e < 8; ++e) dsc = fmaf(qf[e], kf[e], dsc);
+  for (int j = 0; j < 8; ++j) {
+    const int jj = hf * 8 + j;
+    const uint4 qu = *reinterpret_cast<const uint4*>(smem + kPaQ + pa_swz(r, jj));
+    const uint4 ku = *reinterpret_cast<const uint4*>(kt + scr(ti, jj * 8));
+    float qf[8], kf[8];
+    Chunk<__nv_bfloat16>::unpack(qu, qf);
+    Chunk<__nv_bfloat16>::unpack(ku, kf);
+#pragma unroll
+    for (int e = 0; e < 8; ++e) dp = fmaf(qf[e], kf[e], dp);
+  }
+  s_x[hf * kPaRows + r] = dp;
+  s_y[hf * kPaRows + r] = l;
+  __syncthreads();
+  const float dsc = (dp + s_x[(hf ^ 1) * kPaRows + r]) * qscale;  // k~[0] = 0: q[0] drops out
+  const float lt = l + s_y[(hf ^ 1) * kPaRows + r];
+  const float M = fmaxf(m, dsc);
+  const float cO = (m == -INFINITY) ? 0.f : exp2f(m - M);
+  const float cD = exp2f(dsc - M);
+  const float inv = 1.f / (lt * cO + cD);
+  char* orow = a.out + ((size_t)(row_ok ? tau_r : tok0) * L.Hq + (size_t)h * G + r % G) * ROW;
+  for (int c0 = 0; c0 < HALF; c0 += 32) {
+    float f[32];
+    if (ntiles > 0) pa_ld32(tO + lane_base + col0 + c0, f);  // CTA-uniform
+    if (ntiles == 0 || m == -INFINITY) {
+#pragma unroll
+      for (int i = 0; i < 32; ++i) f[i] = 0.f;
     }
-    dsc *= qscale;  // k~[0] = 0, so q[0] drops out
-    const float M = fmaxf(m, dsc);
-    const float cO = (m == -INFINITY) ? 0.f : exp2f(m - M);
-    const float cD = exp2f(dsc - M);
-    const float inv = 1.f / (l * cO + cD);
-    char* orow = a.out + ((size_t)(row_ok ? tau_r : tok0) * L.Hq + (size_t)h * G + r % G) * ROW;
-    for (int c0 = 0; c0 < D; c0 += 32) {
-      float f[32];
-      if (ntiles > 0) pa_ld32(tO + lane_base + c0, f);  // CTA-uniform
-      if (ntiles == 0 || m == -INFINITY) {
+    if (row_ok) {
 #pragma unroll
-        for (int i = 0; i < 32; ++i) f[i] = 0.f;
-      }
-      if (row_ok) {
+      for (int q4 = 0; q4 < 4; ++q4) {
+        const int cc = col0 + c0 + q4 * 8;
+        float vf[8], o[8];
+        Chunk<__nv_bfloat16>::unpack(*reinterpret_cast<const uint4*>(vt + scr(ti, cc)), vf);
 #pragma unroll
-        for (int q4 = 0; q4 < 4; ++q4) {
-          float vf[8], o[8];
-          Chunk<__nv_bfloat16>::unpack(*reinterpret_cast<const uint4*>(vrow + c0 + q4 * 8), vf);
-#pragma unroll
-          for (int e = 0; e < 8; ++e) o[e] = (f[q4 * 8 + e] * cO + vf[e] * cD) * inv;
-          *reinterpret_cast<uint4*>(orow + (c0 + q4 * 8) * 2) = Chunk<__nv_bfloat16>::pack(o);
-        }
+        for (int e = 0; e < 8; ++e) o[e] = (f[q4 * 8 + e] * cO + vf[e] * cD) * inv;
+        *reinterpret_cast<uint4*>(orow + cc * 2) = Chunk<__nv_bfloat16>::pack(o);
       }
     }
   }
