@@ -54,6 +54,10 @@ class Workload:
     cr: tuple                  # ("fixed", CR) | ("choice", (CRs...)) | ("loguniform", lo, hi)
     scale: float
     seed: int = 0
+    # DMC-HardC (in-layer relaxation ablation): decisions and importance
+    # shared by every head of a layer, so all heads of a sequence have the
+    # same segments and lengths
+    hardc: bool = False
 
     @property
     def group(self) -> int:
@@ -87,6 +91,10 @@ WORKLOADS = {
     # long ragged prompts U[1024, 32768], heavy-tailed CR log-uniform in [1, 32]
     "long_ragged": Workload("long_ragged", 32, 8, 32, 32, 128, "bf16",
                             (1024, 32768), 128, ("loguniform", 1.0, 32.0), 0.5),
+    # the 7B 4x shape with DMC-HardC decisions: one alpha and omega per token
+    # for all heads of a layer
+    "llama2_7b_4x_hardc": Workload("llama2_7b_4x_hardc", 32, 32, 32, 32, 128, "bf16",
+                                   (2048, 2048), 512, ("fixed", 4.0), 0.5, hardc=True),
 }
 
 
@@ -141,6 +149,13 @@ def _draw_tokens(n, wl: Workload, p_layer, g, device, want_full_q: bool):
     u = torch.rand((n, H), generator=g, device=device)
     mag = torch.randn((n, H), generator=g, device=device).abs() + 0.1
     p = torch.as_tensor(p_layer, dtype=torch.float32, device=device)
+    if wl.hardc:
+        # one decision and one importance per token for every head of the layer
+        u, mag, p = u[:, :1].expand(n, H), mag[:, :1].expand(n, H), p[:1].expand(H)
+        if want_full_q:
+            q[:, :, 0] = q[:, :1, 0]
+        else:
+            q[:, :] = q[:, :1].clone()
     sign = torch.where(u < p[None, :], -1.0, 1.0)
     k[:, :, 0] = sign * s * mag
     return q, k, v

@@ -1,4 +1,4 @@
-"""The CUDA path at the full sizes of the five large workloads (GPU).
+"""The CUDA path at the full sizes of the large workloads (GPU).
 
 Each case runs the whole workload through the C ABI in the launch
 configuration the benchmark uses (one cache, one launch per layer per decode
@@ -18,7 +18,8 @@ from tests import dmc_harness as H
 
 pytestmark = pytest.mark.gpu
 
-CASES = ["llama2_7b_4x", "llama2_7b_mixed", "llama2_13b_4x", "llama2_70b_gqa_2x", "long_ragged"]
+CASES = ["llama2_7b_4x", "llama2_7b_mixed", "llama2_13b_4x", "llama2_70b_gqa_2x", "long_ragged",
+         "llama2_7b_4x_hardc"]
 
 
 @pytest.mark.parametrize("name", CASES)
@@ -29,6 +30,11 @@ def test_full_size_sampled(cuda_dev, name):
         print(f"{name}: {wl.num_layers} of {S.WORKLOADS[name].num_layers} layers fit the device")
     run = H.Run(wl, cuda_dev, H.random_samples(wl, 64, seed=17), cache=cache)
     assert run.len_ok, run.len_msgs[:5]
+    if wl.hardc:
+        # DMC-HardC: every head of a sequence holds the same number of slots
+        for layer in range(wl.num_layers):
+            ln = cache.lengths(layer)
+            assert bool((ln == ln[:, :1]).all()), layer
     bad = run.compare()
     assert not bad, bad[:10]
     del run, cache
