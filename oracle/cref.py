@@ -27,7 +27,7 @@ class Instance(C.Structure):
         ("K", C.c_void_p), ("V", C.c_void_p), ("z", C.c_void_p),
         ("pK", C.c_void_p), ("pV", C.c_void_p), ("pz", C.c_void_p),
         ("len_prompt", C.c_void_p), ("len_final", C.c_void_p), ("lens", C.c_void_p),
-        ("out", C.c_void_p), ("status", C.c_int32),
+        ("out", C.c_void_p), ("status", C.c_int32), ("window", C.c_int32),
     ]
 
 
@@ -62,7 +62,8 @@ def _ptr(a):
     return a.ctypes.data if a is not None else None
 
 
-def run_heads(heads, threads: int = 1, want_out: bool = True, want_prompt_slots: bool = True):
+def run_heads(heads, threads: int = 1, want_out: bool = True, want_prompt_slots: bool = True,
+              window: int = 0):
     """Run independent head instances.
 
     heads: list of dicts with k_prompt [T,d], v_prompt [T,d], q0_prompt [T,G],
@@ -92,6 +93,7 @@ def run_heads(heads, threads: int = 1, want_out: bool = True, want_prompt_slots:
         keep.append((pk, pv, pq0, dk, dv, dq))
         inst = insts[i]
         inst.d, inst.G, inst.n_prompt, inst.n_decode = d, G, T, S
+        inst.window = int(window)
         inst.pk, inst.pv, inst.pq0 = _ptr(pk), _ptr(pv), _ptr(pq0)
         inst.dk, inst.dv, inst.dq = _ptr(dk), _ptr(dv), _ptr(dq)
         inst.cap = cap

@@ -13,7 +13,11 @@
  *   accumulate (alpha = 1, cache not empty):
  *       z <- z + omega;  K_l <- (K_l z_prev + k_t omega) / z;  V_l likewise
  *   append otherwise: new slot (k_t, v_t), z = omega
- * and, for decode tokens, softmax attention of every query of the group over
+ * With window = w > 0 (the window-grouping approximation, Sec. 3.3) the last
+ * slot is instead the omega-weighted mean of the last min(segment length, w)
+ * tokens of its segment, z their summed omega: the open segment's last w
+ * tokens are kept and the slot recomputed from them at every merge.
+ * And, for decode tokens, softmax attention of every query of the group over
  * the updated cache, Eq. (attn-softmax), with q[0] removed and scale
  * 1/sqrt(d_h) (masking appendix). Everything is double precision; inputs are
  * float (bf16 and fp32 inputs are exact in float).
@@ -47,7 +51,16 @@ typedef struct {
   int32_t* lens;        /* [n_decode] slots after each decode token (may be NULL) */
   double* out;          /* [n_decode][G][d] attention outputs (may be NULL) */
   int32_t status;       /* 0 ok, 1 capacity exceeded, 2 out of memory */
+  int32_t window;       /* 0: Algorithm 1; w > 0: window grouping over w tokens */
 } dmc_ref_instance;
+
+/* The open segment's last `window` tokens (k with k[0] cleared, v, omega). */
+typedef struct {
+  int w, n;  /* window, tokens of the segment so far */
+  double* k; /* [w][d] ring: token p of the segment at row p % w */
+  double* v;
+  double* om;
+} seg_ring;
 
 static double sigmoid(double x) { return 1.0 / (1.0 + exp(-x)); }
 
@@ -61,8 +74,41 @@ static double importance(const float* q0, int G, int stride) {
 
 /* Algorithm 1 for one token. Returns 0, or 1 when a new slot would not fit. */
 static int update(int d, int cap, double* K, double* V, double* z, int* len,
-                  const float* k, const float* v, double omega) {
+                  const float* k, const float* v, double omega, seg_ring* ring) {
   int alpha = decide((double)k[0]);
+  if (ring) {
+    /* window grouping: record the token, the last slot is the mean of the
+       segment's last w tokens */
+    int open = !(alpha == 1 && *len > 0);
+    if (open) {
+      if (*len >= cap) return 1;
+      ring->n = 0;
+      *len += 1;
+    }
+    int row = ring->n % ring->w;
+    ring->k[(size_t)row * d] = 0.0;
+    for (int i = 1; i < d; ++i) ring->k[(size_t)row * d + i] = (double)k[i];
+    for (int i = 0; i < d; ++i) ring->v[(size_t)row * d + i] = (double)v[i];
+    ring->om[row] = omega;
+    ring->n += 1;
+    int m = ring->n < ring->w ? ring->n : ring->w;
+    double* Kl = K + (size_t)(*len - 1) * d;
+    double* Vl = V + (size_t)(*len - 1) * d;
+    double zs = 0.0;
+    for (int i = 0; i < d; ++i) { Kl[i] = 0.0; Vl[i] = 0.0; }
+    for (int e = 0; e < m; ++e) {
+      int r = (ring->n - 1 - e) % ring->w;
+      double om = ring->om[r];
+      zs += om;
+      for (int i = 0; i < d; ++i) {
+        Kl[i] += om * ring->k[(size_t)r * d + i];
+        Vl[i] += om * ring->v[(size_t)r * d + i];
+      }
+    }
+    for (int i = 0; i < d; ++i) { Kl[i] /= zs; Vl[i] /= zs; }
+    z[*len - 1] = zs;
+    return 0;
+  }
   if (alpha == 1 && *len > 0) {
     int l = *len - 1;
     double z_prev = z[l];
@@ -115,11 +161,20 @@ int dmc_ref_run(dmc_ref_instance* in) {
   double* z = in->z ? in->z : (double*)malloc(sizeof(double) * (size_t)cap);
   double* s = (double*)malloc(sizeof(double) * (size_t)(cap > 0 ? cap : 1));
   int len = 0;
+  seg_ring ring_store, *ring = NULL;
+  memset(&ring_store, 0, sizeof(ring_store));
+  if (in->window > 0) {
+    ring_store.w = in->window;
+    ring_store.k = (double*)malloc(sizeof(double) * (size_t)in->window * d);
+    ring_store.v = (double*)malloc(sizeof(double) * (size_t)in->window * d);
+    ring_store.om = (double*)malloc(sizeof(double) * (size_t)in->window);
+    ring = &ring_store;
+  }
   in->status = 0;
-  if (!K || !V || !z || !s) { in->status = 2; goto done; }
+  if (!K || !V || !z || !s || (ring && (!ring->k || !ring->v || !ring->om))) { in->status = 2; goto done; }
   for (int t = 0; t < in->n_prompt; ++t) {
     double w = importance(in->pq0 + (size_t)t * G, G, 1);
-    if (update(d, cap, K, V, z, &len, in->pk + (size_t)t * d, in->pv + (size_t)t * d, w)) {
+    if (update(d, cap, K, V, z, &len, in->pk + (size_t)t * d, in->pv + (size_t)t * d, w, ring)) {
       in->status = 1; goto done;
     }
   }
@@ -130,7 +185,7 @@ int dmc_ref_run(dmc_ref_instance* in) {
   for (int t = 0; t < in->n_decode; ++t) {
     const float* qt = in->dq + (size_t)t * G * d;
     double w = importance(qt, G, d);
-    if (update(d, cap, K, V, z, &len, in->dk + (size_t)t * d, in->dv + (size_t)t * d, w)) {
+    if (update(d, cap, K, V, z, &len, in->dk + (size_t)t * d, in->dv + (size_t)t * d, w, ring)) {
       in->status = 1; goto done;
     }
     if (in->lens) in->lens[t] = len;
@@ -144,6 +199,9 @@ done:
   if (!in->V) free(V);
   if (!in->z) free(z);
   free(s);
+  free(ring_store.k);
+  free(ring_store.v);
+  free(ring_store.om);
   return in->status;
 }
 

@@ -74,6 +74,9 @@ class HeadCache:
         self.K: list[np.ndarray] = []
         self.V: list[np.ndarray] = []
         self.z: list[float] = []
+        # tokens (k with k[0] cleared, v, omega) of the open segment, for the
+        # window-grouping approximation
+        self.seg: list[tuple] = []
 
     def __len__(self) -> int:
         return len(self.K)
@@ -85,16 +88,34 @@ class HeadCache:
         return K, V, np.array(self.z, dtype=f64)
 
 
-def update(cache: HeadCache, k_t, v_t, alpha_t: int, omega_t: float) -> None:
+def update(cache: HeadCache, k_t, v_t, alpha_t: int, omega_t: float, window: int = 0) -> None:
     """Algorithm 1: single-head KV cache update with DMC.
 
     k_t[0] is cleared first (Algorithm 1, third step). With alpha_t = 1 the
     token is merged into the last slot as the omega-weighted running mean,
     z_t = z_{t-1} + omega_t; with alpha_t = 0 it opens a new slot, z_t = omega_t.
-    An empty cache always receives a new slot."""
+    An empty cache always receives a new slot.
+
+    window = w > 0: the window-grouping approximation (Sec. 3.3), where
+    Eq. partial-accumulation runs over the last w tokens only: the last slot
+    is the omega-weighted mean of the last min(segment length, w) tokens of
+    its segment and z their summed omega."""
     k = np.array(k_t, dtype=f64)
     k[0] = 0.0
     v = np.array(v_t, dtype=f64)
+    if window > 0:
+        if alpha_t == 1 and len(cache) > 0:
+            cache.seg = (cache.seg + [(k, v, float(omega_t))])[-window:]
+            w = np.array([t[2] for t in cache.seg])
+            cache.K[-1] = (w[:, None] * np.array([t[0] for t in cache.seg])).sum(0) / w.sum()
+            cache.V[-1] = (w[:, None] * np.array([t[1] for t in cache.seg])).sum(0) / w.sum()
+            cache.z[-1] = float(w.sum())
+        else:
+            cache.seg = [(k, v, float(omega_t))]
+            cache.K.append(k)
+            cache.V.append(v)
+            cache.z.append(float(omega_t))
+        return
     if alpha_t == 1 and len(cache) > 0:
         z_prev = cache.z[-1]
         z_t = z_prev + omega_t
@@ -123,7 +144,7 @@ def attend(cache: HeadCache, q_t) -> np.ndarray:
     return p @ V
 
 
-def run_head(k_prompt, v_prompt, q0_prompt, k_dec, v_dec, q_dec, cache=None):
+def run_head(k_prompt, v_prompt, q0_prompt, k_dec, v_dec, q_dec, cache=None, window: int = 0):
     """One KV head through a prompt and then decode tokens (formulation A).
 
     k_prompt, v_prompt [T, d]; q0_prompt [T, G] (first neuron of each query of
@@ -144,7 +165,7 @@ def run_head(k_prompt, v_prompt, q0_prompt, k_dec, v_dec, q_dec, cache=None):
         cache = HeadCache(d)
     for t in range(k_prompt.shape[0]):
         update(cache, k_prompt[t], v_prompt[t],
-               int(decision(k_prompt[t, 0])), float(importance(q0_prompt[t])))
+               int(decision(k_prompt[t, 0])), float(importance(q0_prompt[t])), window)
     Kp, Vp, zp = cache.arrays()
     S = k_dec.shape[0]
     G = q_dec.shape[1] if S else 0
@@ -152,7 +173,7 @@ def run_head(k_prompt, v_prompt, q0_prompt, k_dec, v_dec, q_dec, cache=None):
     lens = np.zeros(S, dtype=np.int64)
     for s in range(S):
         update(cache, k_dec[s], v_dec[s],
-               int(decision(k_dec[s, 0])), float(importance(q_dec[s, :, 0])))
+               int(decision(k_dec[s, 0])), float(importance(q_dec[s, :, 0])), window)
         for g in range(G):
             out[s, g] = attend(cache, q_dec[s, g])
         lens[s] = len(cache)
@@ -161,7 +182,7 @@ def run_head(k_prompt, v_prompt, q0_prompt, k_dec, v_dec, q_dec, cache=None):
             "cache": cache}
 
 
-def prompt_attention(k, v, q, cache=None):
+def prompt_attention(k, v, q, cache=None, window: int = 0):
     """Attention outputs of every prompt token at inference (formulation A).
 
     Sec. 3.2 (intermediate compression steps): at inference the last slot
@@ -174,7 +195,7 @@ def prompt_attention(k, v, q, cache=None):
     d = np.asarray(k).shape[1]
     G = np.asarray(q).shape[1]
     empty = np.zeros((0, d))
-    return run_head(empty, empty, np.zeros((0, G)), k, v, q, cache=cache)["out"]
+    return run_head(empty, empty, np.zeros((0, G)), k, v, q, cache=cache, window=window)["out"]
 
 
 def decode_lengths(k0_tokens, start_len: int = 0) -> np.ndarray:
@@ -206,16 +227,24 @@ def segment_ids(k0_tokens) -> np.ndarray:
     return np.cumsum(opens) - 1
 
 
-def segment_slots(k_prompt, v_prompt, q0_prompt):
+def segment_slots(k_prompt, v_prompt, q0_prompt, window: int = 0):
     """Slots of a prompt compressed into an empty cache, as segment means.
 
     K_j = sum_{t in seg j} omega_t k'_t / z_j, V_j likewise, z_j = sum omega_t,
-    where k'_t is k_t with its first component cleared. Returns K, V, z."""
+    where k'_t is k_t with its first component cleared. With window = w > 0
+    (window grouping) only the last min(|seg j|, w) tokens of each segment
+    count. Returns K, V, z."""
     k = np.array(k_prompt, dtype=f64)
     v = np.array(v_prompt, dtype=f64)
     k[:, 0] = 0.0
     seg = segment_ids(np.asarray(k_prompt, dtype=f64)[:, 0])
     w = importance(q0_prompt)
+    if window > 0:
+        # position of each token counted from its segment's end
+        from_end = np.zeros(len(seg), dtype=np.int64)
+        for t in range(len(seg) - 2, -1, -1):
+            from_end[t] = from_end[t + 1] + 1 if seg[t + 1] == seg[t] else 0
+        w = np.where(from_end < window, w, 0.0)
     n = int(seg[-1]) + 1
     z = np.zeros(n, dtype=f64)
     Ks = np.zeros((n, k.shape[1]), dtype=f64)
@@ -257,6 +286,32 @@ def unrolled_states(k, v, q0_group):
     return kt, vt, z, alpha
 
 
+def unrolled_states_window(k, v, q0_group, window: int):
+    """The window-grouping approximation of Eq. partial-accumulation (Sec. 3.3):
+    the state of token i is the recurrence run independently over the window
+    of the last w tokens up to i, started afresh at the window's first token
+    (z = omega, k~ = k there). Same returns as unrolled_states."""
+    k = np.array(k, dtype=f64)
+    v = np.array(v, dtype=f64)
+    alpha = decision(k[:, 0]).astype(f64)
+    k[:, 0] = 0.0
+    w = importance(q0_group)
+    n, d = k.shape
+    kt = np.zeros((n, d), dtype=f64)
+    vt = np.zeros((n, d), dtype=f64)
+    z = np.zeros(n, dtype=f64)
+    for i in range(n):
+        s0 = max(0, i - window + 1)
+        zi, ki, vi = w[s0], k[s0].copy(), v[s0].copy()
+        for j in range(s0 + 1, i + 1):
+            zj = zi * alpha[j] + w[j]
+            ki = (alpha[j] * ki * zi + k[j] * w[j]) / zj
+            vi = (alpha[j] * vi * zi + v[j] * w[j]) / zj
+            zi = zj
+        z[i], kt[i], vt[i] = zi, ki, vi
+    return kt, vt, z, alpha
+
+
 def training_mask(alpha) -> np.ndarray:
     """Additive mask of the masking figure for binary alpha: row i (query),
     column j (state): 0 if j == i, log(1 - alpha_{j+1}) if j < i, -inf if j > i."""
@@ -271,14 +326,17 @@ def training_mask(alpha) -> np.ndarray:
     return M
 
 
-def masked_attention(k, v, q):
+def masked_attention(k, v, q, window: int = 0):
     """Outputs of every token of one sequence, training formulation.
 
     k, v [n, d]; q [n, G, d]. The score of query i against state j is
     q_i[1:]^T k~_j[1:] / sqrt(d_h) + M[i, j] (masking appendix). Returns
     [n, G, d]."""
     q = np.array(q, dtype=f64)
-    kt, vt, _, alpha = unrolled_states(k, v, q[:, :, 0])
+    if window > 0:
+        kt, vt, _, alpha = unrolled_states_window(k, v, q[:, :, 0], window)
+    else:
+        kt, vt, _, alpha = unrolled_states(k, v, q[:, :, 0])
     q[:, :, 0] = 0.0
     M = training_mask(alpha)
     n, G, d = q.shape

@@ -73,3 +73,26 @@ def test_c_oracle_matches_numpy_oracle(G):
         assert np.allclose(c["out"], r["out"], atol=1e-12)
         K, V, z = r["cache"].arrays()
         assert np.allclose(c["K"], K, atol=1e-12) and np.allclose(c["z"], z, atol=1e-12)
+
+
+@pytest.mark.parametrize("window", [1, 4, 12])
+def test_c_oracle_window_grouping_matches_numpy(window):
+    """The C oracle's window grouping against the numpy oracle (prompt then
+    decode with outputs), grouped queries."""
+    rng = np.random.default_rng(90 + window)
+    d, G, T, S_ = 8, 2, 60, 25
+    kp, vp = rng.normal(size=(T, d)), rng.normal(size=(T, d))
+    kp[:, 0] = np.where(rng.random(T) < 0.2, -1.0, 1.0) * (np.abs(kp[:, 0]) + 0.1)
+    q0p = rng.normal(size=(T, G))
+    kd, vd = rng.normal(size=(S_, d)), rng.normal(size=(S_, d))
+    kd[:, 0] = np.where(rng.random(S_) < 0.2, -1.0, 1.0) * (np.abs(kd[:, 0]) + 0.1)
+    qd = rng.normal(size=(S_, G, d))
+    f = lambda a: a.astype(np.float32).astype(np.float64)
+    kp, vp, q0p, kd, vd, qd = map(f, (kp, vp, q0p, kd, vd, qd))
+    ref = R.run_head(kp, vp, q0p, kd, vd, qd, window=window)
+    got = cref.run_heads([{"k_prompt": kp, "v_prompt": vp, "q0_prompt": q0p,
+                           "k_dec": kd, "v_dec": vd, "q_dec": qd}], window=window)[0]
+    assert got["prompt_len"] == ref["prompt_len"] and np.allclose(got["prompt_K"], ref["prompt_K"])
+    K, V, z = ref["cache"].arrays()
+    assert np.allclose(got["K"], K) and np.allclose(got["V"], V) and np.allclose(got["z"], z)
+    assert np.allclose(got["out"], ref["out"], atol=1e-10)

@@ -284,6 +284,60 @@ def test_prompt_attention_all_accumulate_is_running_mean():
     assert np.allclose(R.prompt_attention(k, v, q)[:, 0], want, atol=1e-12)
 
 
+@pytest.mark.parametrize("window", [1, 2, 5, 12])
+def test_window_grouping_sequential_equals_training_mask(window):
+    """Window grouping (Sec. 3.3): token-by-token updates over the last w
+    tokens of a segment give the same outputs as the training formulation,
+    where each token's state is the recurrence re-run over its last w tokens."""
+    rng = np.random.default_rng(11 + window)
+    n, d = 40, 6
+    k, v = rng.normal(size=(n, d)), rng.normal(size=(n, d))
+    k[:, 0] = np.where(rng.random(n) < 0.2, -1.0, 1.0) * (np.abs(k[:, 0]) + 0.1)  # long segments
+    q = rng.normal(size=(n, 2, d))
+    got = R.prompt_attention(k, v, q, window=window)
+    assert np.allclose(got, R.masked_attention(k, v, q, window=window), atol=1e-12)
+
+
+@pytest.mark.parametrize("window", [1, 3, 7])
+def test_window_grouping_slots_are_means_of_the_last_w_tokens(window):
+    rng = np.random.default_rng(21 + window)
+    n, d = 50, 5
+    k, v = rng.normal(size=(n, d)), rng.normal(size=(n, d))
+    k[:, 0] = np.where(rng.random(n) < 0.15, -1.0, 1.0) * (np.abs(k[:, 0]) + 0.1)
+    q0 = rng.normal(size=(n, 1))
+    r = R.run_head(k, v, q0, np.zeros((0, d)), np.zeros((0, d)), np.zeros((0, 1, d)), window=window)
+    K, V, z = R.segment_slots(k, v, q0, window=window)
+    assert np.allclose(r["prompt_K"], K) and np.allclose(r["prompt_V"], V) and np.allclose(r["prompt_z"], z)
+    # brute force for every slot: the last min(len, w) tokens of its segment
+    seg = R.segment_ids(k[:, 0])
+    om = R.importance(q0)
+    kk = k.copy()
+    kk[:, 0] = 0.0
+    for j in range(int(seg[-1]) + 1):
+        idx = np.nonzero(seg == j)[0][-window:]
+        assert np.allclose(K[j], (om[idx, None] * kk[idx]).sum(0) / om[idx].sum())
+        assert np.isclose(z[j], om[idx].sum())
+
+
+def test_window_grouping_wide_window_is_exact_dmc():
+    rng = np.random.default_rng(31)
+    n, d = 30, 4
+    k, v, q = rng.normal(size=(n, d)), rng.normal(size=(n, d)), rng.normal(size=(n, 1, d))
+    assert np.allclose(R.prompt_attention(k, v, q, window=n), R.prompt_attention(k, v, q), atol=1e-12)
+
+
+def test_window_one_keeps_only_the_last_token():
+    """w = 1: each slot is its segment's last token, z its omega."""
+    rng = np.random.default_rng(41)
+    n, d = 20, 4
+    k, v = rng.normal(size=(n, d)), rng.normal(size=(n, d))
+    q0 = rng.normal(size=(n, 1))
+    K, V, z = R.segment_slots(k, v, q0, window=1)
+    seg = R.segment_ids(k[:, 0])
+    last = [int(np.nonzero(seg == j)[0][-1]) for j in range(int(seg[-1]) + 1)]
+    assert np.allclose(V, v[last]) and np.allclose(z, R.importance(q0)[last])
+
+
 def test_gqa_equal_group_q0_reduces_to_mha_omega():
     rng = _rng(11)
     n, d, G = 20, 6, 4
