@@ -75,7 +75,11 @@ typedef struct {
   int32_t max_slots_per_head;  /* slot capacity of one head (page-table width) */
   int64_t num_pages;           /* pages in the pool shared by all layers and heads */
   int32_t max_prefill_tokens;  /* largest total_tokens of one dmc_prefill_compress */
-  int32_t reserved;            /* must be 0 */
+  int32_t window;              /* 0: DMC as in Algorithm 1. w in [1, 32]: the window-
+                                  grouping approximation (Sec. 3.3): a slot is the
+                                  omega-weighted mean of the last min(segment length,
+                                  w) tokens of its segment; each head then keeps its
+                                  open segment's last tokens (the window cache). */
 } dmc_cache_config;
 
 typedef struct dmc_cache* dmc_cache_t;

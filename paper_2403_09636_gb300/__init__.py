@@ -40,7 +40,7 @@ class dmc_cache_config(C.Structure):
                 ("num_kv_heads", C.c_int32), ("head_dim", C.c_int32), ("dtype", C.c_int32),
                 ("page_size", C.c_int32), ("max_slots_per_head", C.c_int32),
                 ("num_pages", C.c_int64), ("max_prefill_tokens", C.c_int32),
-                ("reserved", C.c_int32)]
+                ("window", C.c_int32)]
 
 
 class DmcError(RuntimeError):
@@ -164,7 +164,8 @@ class DmcCache:
     methods must be contiguous, on the cache's device, in the cache dtype."""
 
     def __init__(self, num_layers, batch, num_q_heads, num_kv_heads, head_dim, dtype,
-                 max_slots_per_head, num_pages, max_prefill_tokens=0, device=None, stream=None):
+                 max_slots_per_head, num_pages, max_prefill_tokens=0, device=None, stream=None,
+                 window=0):
         import torch
         self.torch = torch
         self.device = torch.device(device if device is not None else "cuda")
@@ -172,7 +173,7 @@ class DmcCache:
         self.dtype = dtype
         self.cfg = dmc_cache_config(num_layers, batch, num_q_heads, num_kv_heads, head_dim, tdt,
                                     PAGE_SIZE, max_slots_per_head, int(num_pages),
-                                    int(max_prefill_tokens), 0)
+                                    int(max_prefill_tokens), int(window))
         self.nbytes = dmc_cache_required_bytes(self.cfg)
         if self.nbytes == 0:
             raise DmcError(DMC_ERR_INVALID_ARG, "dmc_cache_required_bytes")

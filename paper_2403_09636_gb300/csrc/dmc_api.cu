@@ -65,7 +65,7 @@ bool valid_config(const dmc_cache_config* c) {
   if (c->dtype != DMC_F32 && c->dtype != DMC_BF16) return false;
   if (c->page_size != dmc::kPage) return false;
   if (c->max_slots_per_head < 1 || c->num_pages < 1 || c->num_pages > (int64_t)INT32_MAX) return false;
-  if (c->max_prefill_tokens < 0 || c->reserved != 0) return false;
+  if (c->max_prefill_tokens < 0 || c->window < 0 || c->window > dmc::kMaxWindow) return false;
   const int64_t nh = (int64_t)c->batch * c->num_kv_heads;
   if (nh * G > dmc::kMaxVirtualHeads) return false;
   return true;
@@ -74,7 +74,7 @@ bool valid_config(const dmc_cache_config* c) {
 // Byte offsets of every region; returns the total size.
 struct Offsets {
   size_t pages, z, ptab, meta, lengths, ctl, counters, pool_top, error, meta_end, partials,
-      pending, pending_at, pending_z, opens, plan, carry, total;
+      pending, pending_at, pending_z, opens, plan, carry, ring, ring_w, seglen, total;
   int MPH, plan_stride;
 };
 
@@ -95,6 +95,7 @@ Offsets offsets(const dmc_cache_config* c) {
   o.lengths = at; at = align_up(at + (size_t)c->num_layers * 2 * NH * 4);
   o.ctl = at; at = align_up(at + (size_t)c->num_layers * 4 * 4);
   o.counters = at; at = align_up(at + (size_t)c->num_layers * NH * G * 4);
+  o.seglen = at; at = align_up(at + (c->window > 0 ? (size_t)c->num_layers * 2 * NH * 4 : 0));
   o.pool_top = at; at = align_up(at + 8);
   o.error = at; at = align_up(at + 4);
   o.meta_end = at;
@@ -105,6 +106,8 @@ Offsets offsets(const dmc_cache_config* c) {
   o.opens = at; at = align_up(at + (size_t)c->max_prefill_tokens * c->num_kv_heads);
   o.plan = at; at = align_up(at + (size_t)c->num_kv_heads * o.plan_stride * 4);
   o.carry = at; at = align_up(at + (size_t)o.plan_stride * c->num_kv_heads * (2 * c->head_dim + 1) * 4);
+  o.ring = at; at = align_up(at + (size_t)c->num_layers * NH * c->window * 2 * row);
+  o.ring_w = at; at = align_up(at + (size_t)c->num_layers * NH * c->window * 4);
   o.total = at;
   return o;
 }
@@ -200,6 +203,10 @@ dmc_status dmc_cache_create(const dmc_cache_config* cfg, void* arena_dev, size_t
   L.plan = reinterpret_cast<int*>(base + o.plan);
   L.plan_stride = o.plan_stride;
   c->carry = reinterpret_cast<float*>(base + o.carry);
+  L.window = cfg->window;
+  L.ring = cfg->window > 0 ? base + o.ring : nullptr;
+  L.ring_w = cfg->window > 0 ? reinterpret_cast<float*>(base + o.ring_w) : nullptr;
+  L.seglen = cfg->window > 0 ? reinterpret_cast<int*>(base + o.seglen) : nullptr;
   L.max_prefill_tokens = cfg->max_prefill_tokens;
   c->meta = base + o.meta;
   c->meta_bytes = o.meta_end - o.meta;
@@ -269,7 +276,7 @@ dmc_status dmc_prefill_attention(dmc_cache_t c, int32_t layer, int32_t first_seq
                                  cudaStream_t stream) {
   if (!c) return DMC_ERR_INVALID_ARG;
   const Layout& L = c->lay;
-  if (!dmc::prefill_attn_supported(L)) return DMC_ERR_INVALID_ARG;
+  if (!dmc::prefill_attn_supported(L) || L.window != 0) return DMC_ERR_INVALID_ARG;
   if (layer < 0 || layer >= L.L || first_seq < 0 || num_seqs < 0 || first_seq + num_seqs > L.B)
     return DMC_ERR_INVALID_ARG;
   if (total_tokens < 0 || total_tokens > L.max_prefill_tokens || max_seqlen < 0 ||

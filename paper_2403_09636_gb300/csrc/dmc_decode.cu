@@ -186,7 +186,8 @@ __device__ __noinline__ void combine_partials(const float* partials, int wf, int
   }
 }
 
-template <typename T, int D>
+// kWin: the cache uses the window-grouping approximation (L.window > 0)
+template <typename T, int D, bool kWin>
 __global__ void __launch_bounds__(kDecodeThreads, 2)
 dmc_decode_kernel(const DecodeArgs a) {
   using G_ = DecodeGeom<T, D>;
@@ -404,7 +405,22 @@ dmc_decode_kernel(const DecodeArgs a) {
         if (accum || len_old % kPage != 0) tgt = pt_row[(len_old - 1) / kPage];
         float zold = 0.f, znew = omega;
         const char* orow = nullptr;
-        if (accum) {
+        // window grouping: the slot is the mean of the segment's last W
+        // tokens, the W - 1 before this one being in the head's ring
+        const int W = kWin ? L.window : 0;
+        const int Wm = kWin ? L.window : 1;  // the ring's modulus (only used when W > 0)
+        int n_old = 0, nwin = 0;  // tokens before this one, of them in the window
+        const char* ring = nullptr;
+        const float* ring_w = nullptr;
+        if (W > 0) {
+          ring = L.ring + ((size_t)a.layer * L.NH + bh) * W * 2 * ROW;
+          ring_w = L.ring_w + ((size_t)a.layer * L.NH + bh) * W;
+          if (accum) {
+            n_old = L.seglen[((size_t)a.layer * 2 + parity) * L.NH + bh];
+            nwin = min(n_old, W - 1);
+            for (int e = 0; e < nwin; ++e) znew += ring_w[(n_old - 1 - e) % Wm];
+          }
+        } else if (accum) {
           orow = L.pages + (size_t)tgt * L.page_bytes + (size_t)((len_old - 1) % kPage) * ROW;
           zold = L.z[(size_t)tgt * kPage + (len_old - 1) % kPage];
           znew = zold + omega;
@@ -418,7 +434,28 @@ dmc_decode_kernel(const DecodeArgs a) {
           CK::unpack(__ldg(reinterpret_cast<const uint4*>(a.v + (size_t)bh * ROW + c * 128 + l8 * 16)), vin);
           if (c == 0 && l8 == 0) kin[0] = 0.f;  // k[0] <- 0 (Algorithm 1)
           float kn[EPC], vn[EPC];
-          if (accum) {
+          if (W > 0) {
+#pragma unroll
+            for (int e = 0; e < EPC; ++e) { kn[e] = kin[e] * omega; vn[e] = vin[e] * omega; }
+            for (int e2 = 0; e2 < nwin; ++e2) {
+              const int pos = (n_old - 1 - e2) % Wm;
+              const float w = ring_w[pos];
+              float ko[EPC], vo[EPC];
+              CK::unpack(*reinterpret_cast<const uint4*>(ring + (size_t)pos * 2 * ROW + c * 128 + l8 * 16), ko);
+              CK::unpack(*reinterpret_cast<const uint4*>(ring + (size_t)pos * 2 * ROW + ROW + c * 128 + l8 * 16), vo);
+#pragma unroll
+              for (int e = 0; e < EPC; ++e) { kn[e] = fmaf(w, ko[e], kn[e]); vn[e] = fmaf(w, vo[e], vn[e]); }
+            }
+#pragma unroll
+            for (int e = 0; e < EPC; ++e) { kn[e] /= znew; vn[e] /= znew; }
+            if (vh % Gv == 0) {
+              // the new token joins the ring at entry n_old % W (no reader of
+              // this launch looks there)
+              char* re = L.ring + ((size_t)a.layer * L.NH + bh) * W * 2 * ROW + (size_t)(n_old % Wm) * 2 * ROW;
+              *reinterpret_cast<uint4*>(re + c * 128 + l8 * 16) = CK::pack(kin);
+              *reinterpret_cast<uint4*>(re + ROW + c * 128 + l8 * 16) = CK::pack(vin);
+            }
+          } else if (accum) {
             float ko[EPC], vo[EPC];
             CK::unpack(*reinterpret_cast<const uint4*>(orow + c * 128 + l8 * 16), ko);
             CK::unpack(*reinterpret_cast<const uint4*>(orow + (size_t)kPage * ROW + c * 128 + l8 * 16), vo);
@@ -478,6 +515,10 @@ dmc_decode_kernel(const DecodeArgs a) {
               L.z[(size_t)page * kPage + slot % kPage] = znew;
             }
             len_nxt[bh] = ok ? slot + 1 : len_old;
+            if (W > 0) {
+              L.ring_w[((size_t)a.layer * L.NH + bh) * W + n_old % Wm] = omega;
+              L.seglen[((size_t)a.layer * 2 + (parity ^ 1)) * L.NH + bh] = n_old + 1;
+            }
             if (flags & kFlagNaN) atomicOr(L.error, DMC_FAULT_NAN_GATE);
           }
         }
@@ -650,12 +691,19 @@ static cudaError_t setup_decode(int nvh, DecodePlan* plan) {
   plan->stages = kRing;
   plan->smem = G_::smem_bytes(nvh);
   if (plan->smem > (size_t)optin) return cudaErrorInvalidConfiguration;
-  e = cudaFuncSetAttribute(dmc_decode_kernel<T, D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  e = cudaFuncSetAttribute(dmc_decode_kernel<T, D, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                            (int)plan->smem);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(dmc_decode_kernel<T, D, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)plan->smem);
   if (e != cudaSuccess) return e;
-  int occ = 0;
-  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, dmc_decode_kernel<T, D>, kDecodeThreads,
+  int occ = 0, occw = 0;
+  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, dmc_decode_kernel<T, D, false>, kDecodeThreads,
                                                     plan->smem);
+  if (e == cudaSuccess)
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occw, dmc_decode_kernel<T, D, true>,
+                                                      kDecodeThreads, plan->smem);
+  occ = min(occ, occw);
   if (e != cudaSuccess) return e;
   if (occ < 1) return cudaErrorInvalidConfiguration;
   plan->grid = min(sms * occ, kMaxDecodeBlocks);
@@ -691,7 +739,8 @@ static cudaError_t launch_decode(const DecodeArgs& a, const DecodePlan& plan, bo
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = pdl ? 1 : 0;
-  return cudaLaunchKernelEx(&cfg, dmc_decode_kernel<T, D>, a);
+  if (a.lay.window > 0) return cudaLaunchKernelEx(&cfg, dmc_decode_kernel<T, D, true>, a);
+  return cudaLaunchKernelEx(&cfg, dmc_decode_kernel<T, D, false>, a);
 }
 
 cudaError_t decode_launch(const Layout& L, int layer, int Gv, const DecodePlan& plan, bool pdl,

@@ -79,7 +79,8 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   return *reinterpret_cast<uint32_t*>(&h);
 }
 
-template <int D>
+// kWin: the cache uses the window-grouping approximation (L.window > 0)
+template <int D, bool kWin>
 __global__ void __launch_bounds__(kGThreads, 1) dmc_decode_gqa_kernel(const GqaArgs a) {
   using G_ = GqaGeom<D>;
   constexpr int ROW = G_::ROW, CPR = G_::CPR, KT = G_::KT;
@@ -324,8 +325,26 @@ __global__ void __launch_bounds__(kGThreads, 1) dmc_decode_gqa_kernel(const GqaA
         const int* pt_row = ptab + (size_t)vh * L.MPH;
         int tgt = -1;
         if (accum || len_old % kPage != 0) tgt = pt_row[(len_old - 1) / kPage];
-        const float zold = accum ? L.z[(size_t)tgt * kPage + (len_old - 1) % kPage] : 0.f;
-        const float znew = accum ? zold + omega : omega;
+        // window grouping: the slot is the mean of the segment's last W tokens,
+        // the W - 1 before this one being in the head's ring
+        const int W = kWin ? L.window : 0;
+        const int Wm = kWin ? L.window : 1;
+        int n_old = 0, nwin = 0;  // tokens before this one, of them in the window
+        const char* ring = nullptr;
+        const float* ring_w = nullptr;
+        float zold = 0.f, znew = omega;
+        if (W > 0) {
+          ring = L.ring + ((size_t)a.layer * NH + vh) * W * 2 * ROW;
+          ring_w = L.ring_w + ((size_t)a.layer * NH + vh) * W;
+          if (accum) {
+            n_old = L.seglen[((size_t)a.layer * 2 + parity) * NH + vh];
+            nwin = min(n_old, W - 1);
+            for (int e = 0; e < nwin; ++e) znew += ring_w[(n_old - 1 - e) % Wm];
+          }
+        } else if (accum) {
+          zold = L.z[(size_t)tgt * kPage + (len_old - 1) % kPage];
+          znew = zold + omega;
+        }
         const bool is_v = lane >= CPR;
         const int c = is_v ? lane - CPR : lane;
         const bool act = lane < 2 * CPR;
@@ -335,7 +354,23 @@ __global__ void __launch_bounds__(kGThreads, 1) dmc_decode_gqa_kernel(const GqaA
           const char* src_in = (is_v ? a.v : a.k) + (size_t)vh * ROW + c * 16;
           CK::unpack(__ldg(reinterpret_cast<const uint4*>(src_in)), in);
           if (!is_v && c == 0) in[0] = 0.f;  // k[0] <- 0 (Algorithm 1)
-          if (accum) {
+          if (W > 0) {
+#pragma unroll
+            for (int e = 0; e < 8; ++e) nw[e] = in[e] * omega;
+            for (int e2 = 0; e2 < nwin; ++e2) {
+              const int pos = (n_old - 1 - e2) % Wm;
+              float old[8];
+              CK::unpack(*reinterpret_cast<const uint4*>(ring + (size_t)pos * 2 * ROW + (is_v ? ROW : 0) + c * 16), old);
+              const float w = ring_w[pos];
+#pragma unroll
+              for (int e = 0; e < 8; ++e) nw[e] = fmaf(w, old[e], nw[e]);
+            }
+#pragma unroll
+            for (int e = 0; e < 8; ++e) nw[e] /= znew;
+            // the new token joins the ring at entry n_old % W
+            char* re = L.ring + ((size_t)a.layer * NH + vh) * W * 2 * ROW + (size_t)(n_old % Wm) * 2 * ROW;
+            *reinterpret_cast<uint4*>(re + (is_v ? ROW : 0) + c * 16) = CK::pack(in);
+          } else if (accum) {
             const char* orow = L.pages + (size_t)tgt * L.page_bytes +
                                (size_t)(is_v ? kPage : 0) * ROW + (size_t)((len_old - 1) % kPage) * ROW;
             float old[8];
@@ -369,6 +404,10 @@ __global__ void __launch_bounds__(kGThreads, 1) dmc_decode_gqa_kernel(const GqaA
           if (slot >= L.max_slots) atomicOr(L.error, DMC_FAULT_SLOT_CAPACITY);
           if (ok) L.z[(size_t)page * kPage + slot % kPage] = znew;
           len_nxt[vh] = ok ? slot + 1 : len_old;
+          if (W > 0) {
+            L.ring_w[((size_t)a.layer * NH + vh) * W + n_old % Wm] = omega;
+            L.seglen[((size_t)a.layer * 2 + (parity ^ 1)) * NH + vh] = n_old + 1;
+          }
           if (flags & kGFlagNaN) atomicOr(L.error, DMC_FAULT_NAN_GATE);
         }
         if (ok && act) {
@@ -518,12 +557,19 @@ static cudaError_t setup_gqa(const Layout& L, DecodePlan* plan) {
   plan->stages = kGRing;
   plan->smem = G_::smem_bytes(L.NH);
   if (plan->smem > (size_t)optin) return cudaErrorInvalidConfiguration;
-  e = cudaFuncSetAttribute(dmc_decode_gqa_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  e = cudaFuncSetAttribute(dmc_decode_gqa_kernel<D, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                            (int)plan->smem);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(dmc_decode_gqa_kernel<D, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)plan->smem);
   if (e != cudaSuccess) return e;
-  int occ = 0;
-  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, dmc_decode_gqa_kernel<D>, kGThreads,
+  int occ = 0, occw = 0;
+  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, dmc_decode_gqa_kernel<D, false>, kGThreads,
                                                     plan->smem);
+  if (e == cudaSuccess)
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occw, dmc_decode_gqa_kernel<D, true>, kGThreads,
+                                                      plan->smem);
+  occ = min(occ, occw);
   if (e != cudaSuccess) return e;
   if (occ < 1) return cudaErrorInvalidConfiguration;
   plan->grid = min(sms * occ, kGMaxBlocks);
@@ -564,8 +610,11 @@ cudaError_t gqa_launch(const Layout& L, int layer, const DecodePlan& plan, bool 
   cfg.attrs = attr;
   cfg.numAttrs = pdl ? 1 : 0;
   cudaError_t e = cudaErrorInvalidValue;
-  if (L.D == 64) e = cudaLaunchKernelEx(&cfg, dmc_decode_gqa_kernel<64>, a);
-  if (L.D == 128) e = cudaLaunchKernelEx(&cfg, dmc_decode_gqa_kernel<128>, a);
+  const bool win = L.window > 0;
+  if (L.D == 64) e = win ? cudaLaunchKernelEx(&cfg, dmc_decode_gqa_kernel<64, true>, a)
+                         : cudaLaunchKernelEx(&cfg, dmc_decode_gqa_kernel<64, false>, a);
+  if (L.D == 128) e = win ? cudaLaunchKernelEx(&cfg, dmc_decode_gqa_kernel<128, true>, a)
+                          : cudaLaunchKernelEx(&cfg, dmc_decode_gqa_kernel<128, false>, a);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }

@@ -12,6 +12,7 @@ namespace dmc {
 constexpr int kPage = 32;              // slots per page (the paper's page size)
 constexpr int kPrefillChunk = 128;     // prompt tokens per prefill block
 constexpr int kMaxVirtualHeads = 16384;
+constexpr int kMaxWindow = 32;         // longest window of the window-grouping approximation
 
 // Device-side view of one cache. Passed by value to every kernel.
 struct Layout {
@@ -39,6 +40,11 @@ struct Layout {
   int* plan;               // [Hkv][plan_stride]: first slot index per prompt chunk
   int plan_stride;
   int max_prefill_tokens;
+  // window grouping (window > 0): the open segment's last tokens per head
+  int window;              // 0 = exact DMC
+  char* ring;              // [L][NH][window][2][D]: token p of the segment at entry p % window
+  float* ring_w;           // [L][NH][window]: its omega
+  int* seglen;             // [L][2][NH]: tokens of the open segment, double-buffered like lengths
 };
 
 __host__ __device__ inline int ceil_div(int a, int b) { return (a + b - 1) / b; }

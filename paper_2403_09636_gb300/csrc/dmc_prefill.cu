@@ -149,7 +149,7 @@ __device__ __forceinline__ float* carry_at(const PrefillArgs& a, int t0, int cs,
 
 template <typename T, int D>
 __device__ __forceinline__ void scan_segment(const PrefillArgs& a, int h, int bh, int tb, int te,
-                                             int slot, bool merge_old, int t0, int s) {
+                                             int slot, bool merge_old, int t0, int s, int t1) {
   using CK = Chunk<T>;
   constexpr int ROW = D * (int)sizeof(T);
   constexpr int LPR = ROW / 16;  // lanes per row
@@ -165,19 +165,53 @@ __device__ __forceinline__ void scan_segment(const PrefillArgs& a, int h, int bh
   char* kdst = L.pages + (size_t)page * L.page_bytes + (size_t)(slot % kPage) * ROW + lr * 16;
   char* vdst = kdst + (size_t)kPage * ROW;
   float* zp = L.z + (size_t)page * kPage + slot % kPage;
+  // Window grouping (W > 0): the slot is the mean of the segment's last W
+  // tokens only; the head's open segment keeps its last W - 1 tokens in the
+  // ring (token p of the segment at entry p % W) and its length in seglen.
+  const int W = L.window;
+  int* seglen = nullptr;
+  char* ring = nullptr;
+  float* ring_w = nullptr;
+  int n_old = 0;  // tokens of the continued segment before this prompt
+  if (W > 0) {
+    const int parity = *reinterpret_cast<const volatile int*>(&L.ctl[a.layer * 4]);
+    seglen = L.seglen + ((size_t)a.layer * 2 + parity) * L.NH + bh;
+    ring = L.ring + ((size_t)a.layer * L.NH + bh) * W * 2 * ROW;
+    ring_w = L.ring_w + ((size_t)a.layer * L.NH + bh) * W;
+    if (merge_old) n_old = *seglen;
+  }
+  const int sb = W > 0 ? max(tb, te - W) : tb;  // first token the slot counts
   if (merge_old && sub == 0) {
-    // the prompt continues the head's last slot: its K z_old, V z_old and
-    // z_old join the sums (one copy, in the first row group's lanes)
-    float ko[EPC], vo[EPC];
-    CK::unpack(*reinterpret_cast<const uint4*>(kdst), ko);
-    CK::unpack(*reinterpret_cast<const uint4*>(vdst), vo);
-    const float zo = *zp;
+    if (W == 0) {
+      // the prompt continues the head's last slot: its K z_old, V z_old and
+      // z_old join the sums (one copy, in the first row group's lanes)
+      float ko[EPC], vo[EPC];
+      CK::unpack(*reinterpret_cast<const uint4*>(kdst), ko);
+      CK::unpack(*reinterpret_cast<const uint4*>(vdst), vo);
+      const float zo = *zp;
 #pragma unroll
-    for (int e = 0; e < EPC; ++e) {
-      ak[e] = ko[e] * zo;
-      av[e] = vo[e] * zo;
+      for (int e = 0; e < EPC; ++e) {
+        ak[e] = ko[e] * zo;
+        av[e] = vo[e] * zo;
+      }
+      zs = lr == 0 ? zo : 0.f;
+    } else {
+      // the continued segment's tokens still inside the window, from the ring
+      const int m = min(n_old, max(0, W - (te - tb)));
+      for (int e = 0; e < m; ++e) {
+        const int pos = (n_old - 1 - e) % W;
+        float ko[EPC], vo[EPC];
+        CK::unpack(*reinterpret_cast<const uint4*>(ring + (size_t)pos * 2 * ROW + lr * 16), ko);
+        CK::unpack(*reinterpret_cast<const uint4*>(ring + (size_t)pos * 2 * ROW + ROW + lr * 16), vo);
+        const float w = ring_w[pos];
+#pragma unroll
+        for (int e2 = 0; e2 < EPC; ++e2) {
+          ak[e2] = fmaf(w, ko[e2], ak[e2]);
+          av[e2] = fmaf(w, vo[e2], av[e2]);
+        }
+        if (lr == 0) zs += w;
+      }
     }
-    zs = lr == 0 ? zo : 0.f;
   }
   // Writes the sums so far (all row groups together) as the carry of the chunk
   // starting at token cs.
@@ -211,7 +245,7 @@ __device__ __forceinline__ void scan_segment(const PrefillArgs& a, int h, int bh
   const char* kb = a.k + (size_t)h * ROW + lr * 16;
   const char* vb = a.v + (size_t)h * ROW + lr * 16;
   // the segment in pieces that end at chunk starts (only split when carries are asked for)
-  int pb = tb;
+  int pb = sb;
   while (pb < te) {
     int pe = te;
     if (carry) {
@@ -264,6 +298,44 @@ __device__ __forceinline__ void scan_segment(const PrefillArgs& a, int h, int bh
   if (lr == 0) *zp = zs;
 }
 
+// Window grouping: the head's open segment [tb, te = end of the prompt), which
+// had n_old tokens before this prompt, leaves its last W - 1 tokens (k with
+// k[0] cleared, v, omega) in the ring and its length in seglen. One warp.
+template <typename T, int D>
+__device__ __forceinline__ void fill_ring(const PrefillArgs& a, int h, int bh, int tb, int te,
+                                          int n_old) {
+  constexpr int ROW = D * (int)sizeof(T);
+  constexpr int LPR = ROW / 16;
+  constexpr int RPI = 32 / LPR;
+  const Layout& L = a.lay;
+  const int W = L.window;
+  const int lane = threadIdx.x & 31, sub = lane / LPR, lr = lane % LPR;
+  const int parity = *reinterpret_cast<const volatile int*>(&L.ctl[a.layer * 4]);
+  char* ring = L.ring + ((size_t)a.layer * L.NH + bh) * W * 2 * ROW;
+  float* ring_w = L.ring_w + ((size_t)a.layer * L.NH + bh) * W;
+  const T* qq = reinterpret_cast<const T*>(a.q);
+  const size_t hrow = (size_t)L.Hkv * ROW;
+  for (int t = max(tb, te - (W - 1)) + sub; t < te; t += RPI) {
+    const int pos = (n_old + t - tb) % W;
+    uint4 kr = __ldg(reinterpret_cast<const uint4*>(a.k + (size_t)t * hrow + (size_t)h * ROW + lr * 16));
+    const uint4 vr = __ldg(reinterpret_cast<const uint4*>(a.v + (size_t)t * hrow + (size_t)h * ROW + lr * 16));
+    if (lr == 0) {
+      // k[0] <- 0: the first element of this lane's piece
+      if (sizeof(T) == 2) kr.x &= 0xffff0000u;
+      else kr.x = 0u;
+    }
+    *reinterpret_cast<uint4*>(ring + (size_t)pos * 2 * ROW + lr * 16) = kr;
+    *reinterpret_cast<uint4*>(ring + (size_t)pos * 2 * ROW + ROW + lr * 16) = vr;
+    if (lr == 0) {
+      float y = 0.f;
+      for (int g = 0; g < L.G; ++g)
+        y += Elt<T>::to_f(qq[(size_t)t * a.q_tok + (size_t)(h * L.G + g) * a.q_head]);
+      ring_w[pos] = sigmoidf_(y / (float)L.G);
+    }
+  }
+  if (lane == 0) L.seglen[((size_t)a.layer * 2 + parity) * L.NH + bh] = n_old + (te - tb);
+}
+
 template <typename T, int D>
 __global__ void __launch_bounds__(kScanThreads) dmc_prefill_scan_kernel(const PrefillArgs a) {
   __shared__ int starts[kPrefillChunk];
@@ -310,14 +382,42 @@ __global__ void __launch_bounds__(kScanThreads) dmc_prefill_scan_kernel(const Pr
   for (int it = warp; it < items; it += kScanThreads / 32) {
     if (pre && it == 0) {
       const int te = nstart > 0 ? starts[0] : next;
-      scan_segment<T, D>(a, h, bh, t0, te, base - 1, true, t0, s);
+      scan_segment<T, D>(a, h, bh, t0, te, base - 1, true, t0, s, t1);
     } else {
       const int j = it - (pre ? 1 : 0);
       const int tb = starts[j];
       const int te = (j + 1 < nstart) ? starts[j + 1] : next;
-      scan_segment<T, D>(a, h, bh, tb, te, base + j, false, t0, s);
+      scan_segment<T, D>(a, h, bh, tb, te, base + j, false, t0, s, t1);
     }
   }
+}
+
+// Window grouping: after the scan (which read the old window of continued
+// segments), one block per (sequence, KV head) finds the head's open segment
+// (from the prompt's last opening token, or the whole prompt if it continued
+// the old one) and stores its last W - 1 tokens and its length.
+template <typename T, int D>
+__global__ void __launch_bounds__(kPlanThreads) dmc_prefill_ring_kernel(const PrefillArgs a) {
+  __shared__ int s_last;
+  const Layout& L = a.lay;
+  const int s = blockIdx.x, h = blockIdx.y;
+  const int bh = (a.first_seq + s) * L.Hkv + h;
+  const int tid = threadIdx.x;
+  int t0, t1;
+  if (!seq_bounds(a, s, t0, t1) || t1 == t0) return;
+  if (L.plan[(size_t)h * L.plan_stride + chunk_id(t0, 0, s)] < 0) return;  // the plan failed
+  if (tid == 0) s_last = -1;
+  __syncthreads();
+  for (int b = t1 - kPlanThreads; b + kPlanThreads > t0; b -= kPlanThreads) {
+    const int t = b + tid;
+    if (t >= t0 && L.opens[(size_t)t * L.Hkv + h]) atomicMax(&s_last, t);
+    if (__syncthreads_or(s_last >= 0)) break;
+  }
+  const int last = s_last;
+  if (tid >= 32) return;
+  const int parity = *reinterpret_cast<const volatile int*>(&L.ctl[a.layer * 4]);
+  const int n_old = last >= 0 ? 0 : L.seglen[((size_t)a.layer * 2 + parity) * L.NH + bh];
+  fill_ring<T, D>(a, h, bh, last >= 0 ? last : t0, t1, n_old);
 }
 
 template <typename T, int D>
@@ -334,6 +434,10 @@ static cudaError_t launch_prefill(const PrefillArgs& a, cudaStream_t stream) {
   if (e != cudaSuccess) return e;
   if (max_chunks > 0) {
     dmc_prefill_scan_kernel<T, D><<<dim3(max_chunks, a.lay.Hkv, a.num_seqs), kScanThreads, 0, stream>>>(a);
+    e = cudaGetLastError();
+  }
+  if (e == cudaSuccess && a.lay.window > 0) {
+    dmc_prefill_ring_kernel<T, D><<<dim3(a.num_seqs, a.lay.Hkv), kPlanThreads, 0, stream>>>(a);
     e = cudaGetLastError();
   }
   return e;

@@ -36,7 +36,8 @@ def expected_step_lengths(prev, k0_np):
     return prev + np.where((prev == 0) | (alpha == 0), 1, 0)
 
 
-def cache_for(wl: S.Workload, device, max_slots=None, num_pages=None, max_prefill_tokens=None):
+def cache_for(wl: S.Workload, device, max_slots=None, num_pages=None, max_prefill_tokens=None,
+              window=0):
     lens = S.prompt_lengths(wl)
     if max_slots is None:
         max_slots = int(lens.max()) + wl.decode_steps + 1
@@ -46,7 +47,8 @@ def cache_for(wl: S.Workload, device, max_slots=None, num_pages=None, max_prefil
     if max_prefill_tokens is None:
         max_prefill_tokens = int(lens.sum())
     return DmcCache(wl.num_layers, wl.batch, wl.num_q_heads, wl.num_kv_heads, wl.head_dim,
-                    wl.torch_dtype, max_slots, num_pages, max_prefill_tokens, device=device)
+                    wl.torch_dtype, max_slots, num_pages, max_prefill_tokens, device=device,
+                    window=window)
 
 
 def exact_final_lengths(wl: S.Workload, device, steps, p=None):
@@ -112,12 +114,13 @@ class Run:
     them."""
 
     def __init__(self, wl: S.Workload, device, samples, decode_steps=None, cache=None,
-                 check_all_lengths=True):
+                 check_all_lengths=True, window=0):
         self.wl = wl
+        self.window = window
         self.samples = list(samples)
         G, d = wl.group, wl.head_dim
         steps = wl.decode_steps if decode_steps is None else decode_steps
-        self.cache = cache if cache is not None else cache_for(wl, device)
+        self.cache = cache if cache is not None else cache_for(wl, device, window=window)
         p = S.append_prob(wl)
         self.inst = {s: {"k_prompt": None, "k_dec": [], "v_dec": [], "q_dec": [], "out": []}
                      for s in self.samples}
@@ -207,7 +210,7 @@ class Run:
                 "k_prompt": I["k_prompt"], "v_prompt": I["v_prompt"], "q0_prompt": I["q0_prompt"],
                 "k_dec": np.array(I["k_dec"]).reshape(-1, d), "v_dec": np.array(I["v_dec"]).reshape(-1, d),
                 "q_dec": np.array(I["q_dec"]).reshape(-1, G, d)})
-        return dict(zip(self.samples, cref.run_heads(heads, threads=threads)))
+        return dict(zip(self.samples, cref.run_heads(heads, threads=threads, window=self.window)))
 
     def compare(self, tol=None):
         """Returns a list of failure strings (empty = parity)."""

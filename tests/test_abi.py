@@ -37,7 +37,7 @@ def test_library_exports_every_declared_symbol(lib):
 def _cfg(**kw):
     base = dict(num_layers=2, batch=3, num_q_heads=8, num_kv_heads=4, head_dim=128,
                 dtype=P.DMC_BF16, page_size=32, max_slots_per_head=100, num_pages=50,
-                max_prefill_tokens=1000, reserved=0)
+                max_prefill_tokens=1000, window=0)
     base.update(kw)
     return P.dmc_cache_config(*[base[f] for f, _ in P.dmc_cache_config._fields_])
 
@@ -51,7 +51,7 @@ def test_required_bytes_accounts_for_the_page_pool(lib):
 
 @pytest.mark.parametrize("bad", [dict(head_dim=96), dict(page_size=16), dict(num_q_heads=6),
                                  dict(dtype=7), dict(num_layers=0), dict(num_pages=0),
-                                 dict(num_q_heads=132, num_kv_heads=4), dict(reserved=1),
+                                 dict(num_q_heads=132, num_kv_heads=4), dict(window=33), dict(window=-1),
                                  dict(batch=4096, num_kv_heads=8)])
 def test_invalid_configs_need_zero_bytes(lib, bad):
     assert P.dmc_cache_required_bytes(_cfg(**bad)) == 0
