@@ -58,6 +58,8 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--window", type=int, default=0,
+                    help="window-grouping approximation over this many tokens (0: exact DMC)")
     ap.add_argument("--pa-layers", type=int, default=4,
                     help="layers of the prompt-attention measurement (0 skips it)")
     ap.add_argument("--graph", action="store_true",
@@ -275,17 +277,33 @@ def run_ours(args, rank, world, dist):
 
     # ---- exact slot counts (from the decisions) for sizing and byte accounting
     plen = []
+    tail = []  # tokens of each head's open segment after its prompt (window grouping)
     for pr in prompts:
         cu = pr["cu_seqlens"].to(torch.int64)
         neg = (pr["k"][:, :, 0] < 0).to(torch.int64)                   # [T, H]
         csum = torch.cat([torch.zeros_like(neg[:1]), torch.cumsum(neg, 0)])
         first = pr["k"][cu[:-1], :, 0] >= 0                             # first token opens anyway
         plen.append(csum[cu[1:]] - csum[cu[:-1]] + first.to(torch.int64))
+        if args.window > 0:
+            opens = neg.clone()
+            opens[cu[:-1]] = 1
+            pos = torch.arange(neg.shape[0], device=dev)[:, None].expand_as(opens)
+            last_open = torch.cummax(torch.where(opens > 0, pos, -1), 0).values  # [T, H]
+            tail.append(cu[1:, None] - last_open[cu[1:] - 1])
     plen = torch.stack(plen)                                            # [L, B, H]
     app = (kd[:, :, :, :, 0] < 0).to(torch.int64)                      # [S, L, B, H]
     before = plen[None] + torch.cumsum(app, 0) - app                     # len_old per decode step
     final = plen + app.sum(0)
     slots_read = int(before.sum())
+    ring_reads = 0
+    if args.window > 0:
+        # window grouping: a merge reads the min(n, w - 1) earlier tokens of the
+        # open segment from the window cache; n restarts at 1 on an append
+        n = torch.stack(tail).to(torch.int64)                           # [L, B, H]
+        for t in range(steps_dec):
+            a_t = app[t]
+            ring_reads += int(torch.where(a_t > 0, 0, torch.clamp(n, max=args.window - 1)).sum())
+            n = torch.where(a_t > 0, torch.ones_like(n), n + 1)
     # the e2e leg reuses layer 0's prompt for every layer and a ring of decode
     # steps, so it needs its own page count; size the pool for both
     ring = min(16, steps_dec)
@@ -296,7 +314,8 @@ def run_ours(args, rank, world, dist):
     max_slots = int(S.prompt_lengths(wl).max()) + steps_dec + 1
     max_prompt = max(pr["max_seqlen"] for pr in prompts)
     total_prompt = max(int(pr["cu_seqlens"][-1]) for pr in prompts)
-    cache = P.DmcCache(Lr, Bt, Hq, Hk, D, dt, max_slots, pages_needed + 64, total_prompt, device=dev)
+    cache = P.DmcCache(Lr, Bt, Hq, Hk, D, dt, max_slots, pages_needed + 64, total_prompt, device=dev,
+                       window=args.window)
     row = D * esize
     n_dec_launch = steps_dec * Lr
     # algorithmic bytes of all decode launches of one step: every unchanged slot
@@ -307,6 +326,11 @@ def run_ours(args, rank, world, dist):
     dec_bytes = (slots_read * 2 * row + acc_events * (2 * row + 4)
                  + n_dec_launch * n_heads * (2 * row + 2 * row + 4 + 8)
                  + n_dec_launch * Bt * Hq * row * 2)
+    if args.window > 0:
+        # instead of the merged slot's old row and z: the window's rows and
+        # omegas, plus the new token written to the window and its length
+        dec_bytes += -acc_events * (2 * row + 4) + ring_reads * (2 * row + 4) \
+            + n_dec_launch * n_heads * (2 * row + 8)
     pf_tokens = sum(int(pr["cu_seqlens"][-1]) for pr in prompts)
     pf_slots = int(plen.sum())
     pf_bytes = sum(int(pr["cu_seqlens"][-1]) * Hk * (2 * row) + int(pr["cu_seqlens"][-1]) * Hq * esize
@@ -419,6 +443,7 @@ def run_ours(args, rank, world, dist):
                    "global_batch": Bt * world, "seq_len": int(S.prompt_lengths(wl).max()) + steps_dec,
                    "parallelism": f"replicas{world}",
                    "launch": "cuda_graph" if args.graph else "stream",
+                   "window": args.window,
                    "l2": "inputs larger than L2: each decode launch streams ~"
                          f"{per_launch_bytes / 1e6:.0f} MB of slots, layers rotate"},
         "decode_only_tokens_per_s": job_rate(world, K, Bt * steps_dec, dec_ms),
