@@ -398,7 +398,50 @@ dmc_decode_kernel(const DecodeArgs a) {
             m = mn;
           }
         }
-      } else if (grp == 0) {
+      } else {
+        // Window grouping: the merge averages the open segment's window with
+        // the new token. The four row groups read the window's rows (entries
+        // grp, grp + 4, ... back from the newest) and add their sums.
+        constexpr int WR = kWin ? EPL : 1;
+        float rk[WR], rv[WR], rz = 0.f;
+        int n_old = 0, nwin = 0;  // tokens before this one, of them in the window
+        if constexpr (kWin) {
+#pragma unroll
+          for (int i = 0; i < EPL; ++i) { rk[i] = 0.f; rv[i] = 0.f; }
+          const int W = L.window;
+          if (accum) {
+            n_old = L.seglen[((size_t)a.layer * 2 + parity) * L.NH + bh];
+            nwin = min(n_old, W - 1);
+            const char* ring = L.ring + ((size_t)a.layer * L.NH + bh) * W * 2 * ROW;
+            const float* ring_w = L.ring_w + ((size_t)a.layer * L.NH + bh) * W;
+            for (int e = grp; e < nwin; e += 4) {
+              const int pos = (n_old - 1 - e) % W;
+              const float w = ring_w[pos];
+              rz += w;
+#pragma unroll
+              for (int c = 0; c < NCH; ++c) {
+                float ko[EPC], vo[EPC];
+                CK::unpack(*reinterpret_cast<const uint4*>(ring + (size_t)pos * 2 * ROW + c * 128 + l8 * 16), ko);
+                CK::unpack(*reinterpret_cast<const uint4*>(ring + (size_t)pos * 2 * ROW + ROW + c * 128 + l8 * 16), vo);
+#pragma unroll
+                for (int q = 0; q < EPC; ++q) {
+                  rk[c * EPC + q] = fmaf(w, ko[q], rk[c * EPC + q]);
+                  rv[c * EPC + q] = fmaf(w, vo[q], rv[c * EPC + q]);
+                }
+              }
+            }
+          }
+#pragma unroll
+          for (int off = 8; off < 32; off <<= 1) {
+#pragma unroll
+            for (int i = 0; i < EPL; ++i) {
+              rk[i] += __shfl_xor_sync(0xffffffffu, rk[i], off);
+              rv[i] += __shfl_xor_sync(0xffffffffu, rv[i], off);
+            }
+            rz += __shfl_xor_sync(0xffffffffu, rz, off);
+          }
+        }
+        if (grp == 0) {
         // Algorithm 1 on the new token, in fp32, result rounded to the cache dtype.
         const int* pt_row = ptab + (size_t)bh * L.MPH;
         int tgt = -1;
@@ -409,17 +452,8 @@ dmc_decode_kernel(const DecodeArgs a) {
         // tokens, the W - 1 before this one being in the head's ring
         const int W = kWin ? L.window : 0;
         const int Wm = kWin ? L.window : 1;  // the ring's modulus (only used when W > 0)
-        int n_old = 0, nwin = 0;  // tokens before this one, of them in the window
-        const char* ring = nullptr;
-        const float* ring_w = nullptr;
         if (W > 0) {
-          ring = L.ring + ((size_t)a.layer * L.NH + bh) * W * 2 * ROW;
-          ring_w = L.ring_w + ((size_t)a.layer * L.NH + bh) * W;
-          if (accum) {
-            n_old = L.seglen[((size_t)a.layer * 2 + parity) * L.NH + bh];
-            nwin = min(n_old, W - 1);
-            for (int e = 0; e < nwin; ++e) znew += ring_w[(n_old - 1 - e) % Wm];
-          }
+          znew = omega + rz;
         } else if (accum) {
           orow = L.pages + (size_t)tgt * L.page_bytes + (size_t)((len_old - 1) % kPage) * ROW;
           zold = L.z[(size_t)tgt * kPage + (len_old - 1) % kPage];
@@ -436,18 +470,10 @@ dmc_decode_kernel(const DecodeArgs a) {
           float kn[EPC], vn[EPC];
           if (W > 0) {
 #pragma unroll
-            for (int e = 0; e < EPC; ++e) { kn[e] = kin[e] * omega; vn[e] = vin[e] * omega; }
-            for (int e2 = 0; e2 < nwin; ++e2) {
-              const int pos = (n_old - 1 - e2) % Wm;
-              const float w = ring_w[pos];
-              float ko[EPC], vo[EPC];
-              CK::unpack(*reinterpret_cast<const uint4*>(ring + (size_t)pos * 2 * ROW + c * 128 + l8 * 16), ko);
-              CK::unpack(*reinterpret_cast<const uint4*>(ring + (size_t)pos * 2 * ROW + ROW + c * 128 + l8 * 16), vo);
-#pragma unroll
-              for (int e = 0; e < EPC; ++e) { kn[e] = fmaf(w, ko[e], kn[e]); vn[e] = fmaf(w, vo[e], vn[e]); }
+            for (int e = 0; e < EPC; ++e) {
+              kn[e] = fmaf(kin[e], omega, rk[(c * EPC + e) % WR]) / znew;
+              vn[e] = fmaf(vin[e], omega, rv[(c * EPC + e) % WR]) / znew;
             }
-#pragma unroll
-            for (int e = 0; e < EPC; ++e) { kn[e] /= znew; vn[e] /= znew; }
             if (vh % Gv == 0) {
               // the new token joins the ring at entry n_old % W (no reader of
               // this launch looks there)
@@ -537,6 +563,7 @@ dmc_decode_kernel(const DecodeArgs a) {
           for (int e = 0; e < EPC; ++e) acc[c * EPC + e] = fmaf(acc[c * EPC + e], corr, p * vr[e]);
         }
         m = mn;
+        }
       }
 
       if (owner || k == n - 1) {
