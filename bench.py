@@ -574,10 +574,16 @@ def run_prompt_attention(args, wl, dev, stream, dist):
 
 def run_e2e(args, wl, cache, prompts, qd, kd, vd, outs, steps_dec, dev, stream, L_, barrier, dist,
             world, local):
-    """Per step: H2D of every layer's prompt (one layer's pinned prompt buffer
-    is reused for every layer) and of every decode step's q/k/v (a pinned ring
-    of `ring` distinct steps is reused cyclically), the same C ABI calls, and a
-    D2H read of every layer's attention output of every decode step."""
+    """The whole step through the C ABI with every input coming from pinned
+    host memory and every attention output read back, inside the timed region:
+    each step copies every layer's prompt (one layer's pinned prompt reused for
+    all layers) and every decode step's q/k/v (a pinned ring of `ring`
+    distinct steps reused cyclically), and reads every decode output back into
+    a pinned ring. The copies run on two copy streams, as a server prefetches
+    its next inputs: the next step's prompts while this step decodes, the next
+    decode steps' q/k/v two steps ahead, each step's outputs as soon as they
+    are written; events order every copy against the kernels that use its
+    buffer."""
     import torch
 
     Lr = wl.num_layers
@@ -586,51 +592,96 @@ def run_e2e(args, wl, cache, prompts, qd, kd, vd, outs, steps_dec, dev, stream, 
     hq0 = pr0["q0"].cpu().pin_memory()
     hk = pr0["k"].cpu().pin_memory()
     hv = pr0["v"].cpu().pin_memory()
-    dq0 = torch.empty_like(pr0["q0"])
-    dk = torch.empty_like(pr0["k"])
-    dv = torch.empty_like(pr0["v"])
+    # device prompt buffers, one per layer (the main leg's, overwritten)
+    dq0 = [pr["q0"] for pr in prompts]
+    dk = [pr["k"] for pr in prompts]
+    dv = [pr["v"] for pr in prompts]
     cu = pr0["cu_seqlens"]
     hqd = qd[:ring].cpu().pin_memory()
     hkd = kd[:ring].cpu().pin_memory()
     hvd = vd[:ring].cpu().pin_memory()
-    gq = torch.empty_like(qd[0])
-    gk = torch.empty_like(kd[0])
-    gv = torch.empty_like(vd[0])
+    gq = [torch.empty_like(qd[0]) for _ in range(2)]
+    gk = [torch.empty_like(kd[0]) for _ in range(2)]
+    gv = [torch.empty_like(vd[0]) for _ in range(2)]
+    go = [torch.empty_like(outs) for _ in range(2)]
     hout = torch.empty((ring,) + tuple(outs.shape), dtype=outs.dtype).pin_memory()
     h, sh = cache.handle, stream.cuda_stream
     tot, mx, ns = int(cu[-1]), pr0["max_seqlen"], cu.numel() - 1
     h2d = Lr * (hq0.numel() * hq0.element_size() + hk.numel() * hk.element_size() +
                 hv.numel() * hv.element_size()) + steps_dec * (
-        gq.numel() * gq.element_size() + gk.numel() * gk.element_size() +
-        gv.numel() * gv.element_size())
+        gq[0].numel() * gq[0].element_size() + gk[0].numel() * gk[0].element_size() +
+        gv[0].numel() * gv[0].element_size())
     d2h = steps_dec * outs.numel() * outs.element_size()
 
-    def step():
-        rc = L_.dmc_cache_reset(h, sh)
-        for l in range(Lr):
-            dq0.copy_(hq0, non_blocking=True)
-            dk.copy_(hk, non_blocking=True)
-            dv.copy_(hv, non_blocking=True)
-            rc |= L_.dmc_prefill_compress(h, l, 0, ns, dq0.data_ptr(), dq0.stride(0), dq0.stride(1),
-                                          dk.data_ptr(), dv.data_ptr(), cu.data_ptr(), tot, mx, sh)
-        for t in range(steps_dec):
-            gq.copy_(hqd[t % ring], non_blocking=True)
-            gk.copy_(hkd[t % ring], non_blocking=True)
-            gv.copy_(hvd[t % ring], non_blocking=True)
-            for l in range(Lr):
-                rc |= L_.dmc_decode_step(h, l, gq[l].data_ptr(), gk[l].data_ptr(), gv[l].data_ptr(),
-                                         outs[l].data_ptr(), sh)
-            hout[t % ring].copy_(outs, non_blocking=True)
-        if rc:
-            raise RuntimeError(f"launch failed: {rc}")
+    cs_p = torch.cuda.Stream(dev)   # prompt copies
+    cs_io = torch.cuda.Stream(dev)  # decode inputs and outputs
+    ev = lambda: torch.cuda.Event()
+    ev_pr = [ev() for _ in range(Lr)]   # prompt of layer l landed
+    ev_pf = [ev() for _ in range(Lr)]   # prefill of layer l done with its buffer
+    ev_in = [ev() for _ in range(2)]    # decode inputs of buffer b landed
+    ev_done = [ev() for _ in range(2)]  # decodes of buffer b done (inputs free, outputs ready)
+    ev_d2h = [ev() for _ in range(2)]   # outputs of buffer b read back
 
-    for _ in range(max(1, args.warmup)):
-        step()
+    def copy_prompts():
+        with torch.cuda.stream(cs_p):
+            for l in range(Lr):
+                cs_p.wait_event(ev_pf[l])
+                dq0[l].copy_(hq0, non_blocking=True)
+                dk[l].copy_(hk, non_blocking=True)
+                dv[l].copy_(hv, non_blocking=True)
+                ev_pr[l].record(cs_p)
+
+    def copy_inputs(t, b):
+        with torch.cuda.stream(cs_io):
+            cs_io.wait_event(ev_done[b])
+            gq[b].copy_(hqd[t % ring], non_blocking=True)
+            gk[b].copy_(hkd[t % ring], non_blocking=True)
+            gv[b].copy_(hvd[t % ring], non_blocking=True)
+            ev_in[b].record(cs_io)
+
+    def run(nsteps):
+        # the first step's prompts and first two decode steps' inputs
+        cs_p.wait_stream(stream)
+        cs_io.wait_stream(stream)
+        copy_prompts()
+        copy_inputs(0, 0)
+        copy_inputs(1 % steps_dec, 1)
+        for i in range(nsteps):
+            rc = L_.dmc_cache_reset(h, sh)
+            for l in range(Lr):
+                stream.wait_event(ev_pr[l])
+                rc |= L_.dmc_prefill_compress(h, l, 0, ns, dq0[l].data_ptr(), dq0[l].stride(0),
+                                              dq0[l].stride(1), dk[l].data_ptr(), dv[l].data_ptr(),
+                                              cu.data_ptr(), tot, mx, sh)
+                ev_pf[l].record(stream)
+            if i + 1 < nsteps:
+                copy_prompts()  # the next step's, while this one decodes
+            for t in range(steps_dec):
+                b = t & 1
+                stream.wait_event(ev_in[b])
+                stream.wait_event(ev_d2h[b])  # outputs of two steps ago are read back
+                for l in range(Lr):
+                    rc |= L_.dmc_decode_step(h, l, gq[b][l].data_ptr(), gk[b][l].data_ptr(),
+                                             gv[b][l].data_ptr(), go[b][l].data_ptr(), sh)
+                ev_done[b].record(stream)
+                with torch.cuda.stream(cs_io):
+                    cs_io.wait_event(ev_done[b])
+                    hout[t % ring].copy_(go[b], non_blocking=True)
+                    ev_d2h[b].record(cs_io)
+                last = i + 1 == nsteps and t + 2 >= steps_dec
+                if not last:
+                    # two steps ahead (at the end of a step, the next step's first two)
+                    copy_inputs((t + 2) % steps_dec, b)
+            if rc:
+                raise RuntimeError(f"launch failed: {rc}")
+        stream.wait_stream(cs_p)
+        stream.wait_stream(cs_io)
+
+    run(max(1, args.warmup))
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     barrier()
     e0.record(stream)
-    for _ in range(args.steps):
-        step()
+    run(args.steps)
     e1.record(stream)
     barrier()
     ms = max_over_ranks(dist, [e0.elapsed_time(e1)], dev)[0]
@@ -641,7 +692,8 @@ def run_e2e(args, wl, cache, prompts, qd, kd, vd, outs, steps_dec, dev, stream, 
             "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
             "note": f"pinned host inputs: one layer's prompt reused for all {Lr} layers, a ring of "
                     f"{ring} decode steps reused cyclically; every attention output is read back into a "
-                    f"pinned ring of {ring} steps"}
+                    f"pinned ring of {ring} steps; copies on two side streams overlap the kernels "
+                    "(next step's prompts during this step's decode, decode inputs two steps ahead)"}
 
 
 def main():
