@@ -26,7 +26,6 @@
 namespace dmc {
 
 constexpr int kPlanThreads = 256;
-constexpr int kPlanUnroll = 8;
 constexpr int kScanThreads = 128;
 
 struct PrefillArgs {
@@ -72,28 +71,20 @@ __global__ void __launch_bounds__(kPlanThreads) dmc_prefill_plan_kernel(const Pr
   if (tid == 0) { s_fail = 0; s_nan = 0; }
   __syncthreads();
   const T* kk = reinterpret_cast<const T*>(a.k);
-  // kPlanUnroll tokens per thread and pass: all their k[0] loads are issued first
-  for (int base = 0; base < ntok; base += kPlanThreads * kPlanUnroll) {
-    float x[kPlanUnroll];
-#pragma unroll
-    for (int u = 0; u < kPlanUnroll; ++u) {
-      const int i = base + u * kPlanThreads + tid;
-      x[u] = i < ntok ? Elt<T>::to_f(kk[((size_t)(t0 + i) * L.Hkv + h) * D]) : 0.f;
+  for (int base = 0; base < ntok; base += kPlanThreads) {
+    const int i = base + tid;
+    bool opens = false;
+    if (i < ntok) {
+      const size_t t = (size_t)(t0 + i);
+      const float x = Elt<T>::to_f(kk[(t * L.Hkv + h) * D]);
+      if (x != x) s_nan = 1;
+      // alpha = round(sigmoid(k[0])) = [k[0] >= 0]; alpha = 0 opens a slot,
+      // and so does the first token of an empty head.
+      opens = !(x >= 0.f) || (i == 0 && len_old == 0);
+      L.opens[t * L.Hkv + h] = opens ? 1 : 0;
     }
-#pragma unroll
-    for (int u = 0; u < kPlanUnroll; ++u) {
-      const int b = base + u * kPlanThreads, i = b + tid;
-      bool opens = false;
-      if (i < ntok) {
-        if (x[u] != x[u]) s_nan = 1;
-        // alpha = round(sigmoid(k[0])) = [k[0] >= 0]; alpha = 0 opens a slot,
-        // and so does the first token of an empty head.
-        opens = !(x[u] >= 0.f) || (i == 0 && len_old == 0);
-        L.opens[(size_t)(t0 + i) * L.Hkv + h] = opens ? 1 : 0;
-      }
-      const unsigned bal = __ballot_sync(0xffffffffu, opens);
-      if (lane == 0 && b + warp * 32 < ntok) atomicAdd(&cnt[(b + warp * 32) / kPrefillChunk], __popc(bal));
-    }
+    const unsigned bal = __ballot_sync(0xffffffffu, opens);
+    if (lane == 0 && base + warp * 32 < ntok) atomicAdd(&cnt[(base + warp * 32) / kPrefillChunk], __popc(bal));
   }
   __syncthreads();
   // exclusive scan of the chunk counts (nch <= max_seqlen / 128 + 1)
