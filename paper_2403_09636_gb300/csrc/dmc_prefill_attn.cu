@@ -150,6 +150,9 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
   float* s_x = reinterpret_cast<float*>(smem + kPaMisc + 64 + 1536);   // [2][128] row exchange
   float* s_y = reinterpret_cast<float*>(smem + kPaMisc + 64 + 2560);   // [2][128] row exchange
   unsigned char* s_op = smem + kPaMisc + 64 + 3584;                    // [128] token opens a slot
+  int* s_wc = reinterpret_cast<int*>(smem + kPaMisc + 64 + 3712);      // [4] openings per warp
+  int* s_wf = reinterpret_cast<int*>(smem + kPaMisc + 64 + 3728);      // [4] the warp has one
+  float* s_wz = reinterpret_cast<float*>(smem + kPaMisc + 64 + 3744);  // [4] its last segment's omega sum
 
   const int t0 = a.cu[s], t1 = a.cu[s + 1];
   if (!(t0 >= 0 && t0 <= t1 && t1 <= a.total_tokens && t1 - t0 <= a.max_seqlen)) return;
@@ -167,7 +170,40 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
   const __nv_bfloat16* qg = reinterpret_cast<const __nv_bfloat16*>(a.q);
   const float* carry = a.carry + ((size_t)cid * L.Hkv + h) * (2 * D + 1);
 
-  // ---- per-token decisions, omega and slot counts of the chunk up to the tile end
+  // ---- Q and the first K/V tile start streaming before anything else. The
+  // first tile is read up to min(128, len_final) slots: every slot the head
+  // holds has been written, and the staircase mask hides those a row does not
+  // see; tiles after the first are read up to the slots the tile's rows see.
+  const uint32_t sQ = smem_u32(smem + kPaQ);
+  for (int i = tid; i < kPaRows * 16; i += kPaThreads) {
+    const int rr = i >> 4, j = i & 15;
+    const int tt = tok0 + rr / G;
+    const bool ok = tt < tokN;
+    const char* src = a.q + (((size_t)(ok ? tt : tok0) * L.Hq + (size_t)h * G + rr % G) * ROW) + j * 16;
+    cp_async16_zfill(sQ + pa_swz(rr, j), src, ok);
+  }
+  auto load_kv = [&](int jt, int hi) {
+    const uint32_t sK = smem_u32(smem + kPaK);
+    const uint32_t sV = smem_u32(smem + kPaV);
+    for (int i = tid; i < kPaSlots * 16; i += kPaThreads) {
+      const int rr = i >> 4, j = i & 15;
+      const int slot = jt * kPaSlots + rr;
+      const bool ok = slot < hi;
+      const int page = ok ? ptab[slot / kPage] : 0;
+      const char* src = L.pages + (size_t)page * L.page_bytes + (size_t)(ok ? slot % kPage : 0) * ROW + j * 16;
+      cp_async16_zfill(sK + pa_swz(rr, j), src, ok);
+      cp_async16_zfill(sV + pa_swz(rr, j), src + (size_t)kPage * ROW, ok);
+    }
+  };
+  load_kv(0, min(kPaSlots, len_final));
+  cp_async_commit();
+
+  // ---- per-token decisions, omega, slot counts and 1 / z of the chunk up to
+  // the tile end. z after token i is the omega sum of i's segment so far: from
+  // the segment's opening token, or from the carried sums when no token of the
+  // chunk up to i opens a slot (a segmented prefix sum over the chunk).
+  int incl = 0, seg = 0;
+  float zs = 0.f;
   if (tid < kPrefillChunk) {
     const int tau = a0 + tid;
     int op = 0;
@@ -182,13 +218,27 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
     }
     s_op[tid] = (unsigned char)op;
     s_om[tid] = om;
-    int incl = op;  // openings up to this token, within the warp for now
+    // within the warp for now: openings up to this token, and the omega sum
+    // back to the last opening (seg: one was found)
+    incl = op;
+    seg = op;
+    zs = om;
 #pragma unroll
     for (int off = 1; off < 32; off <<= 1) {
       const int o = __shfl_up_sync(0xffffffffu, incl, off);
-      if (lane >= off) incl += o;
+      const int so = __shfl_up_sync(0xffffffffu, seg, off);
+      const float zo = __shfl_up_sync(0xffffffffu, zs, off);
+      if (lane >= off) {
+        incl += o;
+        if (!seg) zs += zo;
+        seg |= so;
+      }
     }
-    s_len[tid] = incl;
+    if (lane == 31) {
+      s_wc[warp] = incl;
+      s_wf[warp] = seg;
+      s_wz[warp] = zs;
+    }
   }
   if (tid == 0) {
     asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(&bars[0])));
@@ -202,24 +252,21 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
   }
   __syncthreads();
-  int add = base;
-  if (tid < kPrefillChunk)
-    for (int w = 0; w < warp; ++w) add += s_len[w * 32 + 31];
-  if (warp == 4) {
-    // 1 / z of every token of the chunk (the same for all columns): the
-    // segment's summed omega, continuing the carried sums at the chunk start
-    if (lane == 0) {
-      float z = s_op[0] ? 0.f : carry[2 * D];
-      const int n = tokN - a0;
-      for (int i = 0; i < n; ++i) {
-        if (s_op[i]) z = 0.f;
-        z += s_om[i];
-        s_rz[i] = 1.f / z;
+  if (tid < kPrefillChunk) {
+    int add = base;
+    for (int w = 0; w < warp; ++w) add += s_wc[w];
+    s_len[tid] = incl + add;  // slot count after token a0 + tid
+    if (!seg) {
+      // the segment runs in from earlier warps, or from before the chunk
+      bool found = false;
+      for (int w = warp - 1; w >= 0 && !found; --w) {
+        zs += s_wz[w];
+        found = s_wf[w] != 0;
       }
+      if (!found) zs += carry[2 * D];  // no opening in the chunk up to here
     }
+    s_rz[tid] = 1.f / zs;
   }
-  __syncthreads();
-  if (tid < kPrefillChunk) s_len[tid] += add;  // slot count after token a0 + tid
   __syncthreads();
 
   // ---- thread (r, hf): query row r (token tok0 + r / G, query head h G + r % G),
@@ -231,30 +278,6 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
   const int nvis_max = s_len[tokN - 1 - a0] - 1;
   const int vis_hi = min(nvis_max, len_final);          // slots worth loading
   const int ntiles = (vis_hi + kPaSlots - 1) / kPaSlots;
-
-  const uint32_t sQ = smem_u32(smem + kPaQ);
-  for (int i = tid; i < kPaRows * 16; i += kPaThreads) {
-    const int rr = i >> 4, j = i & 15;
-    const int tt = tok0 + rr / G;
-    const bool ok = tt < tokN;
-    const char* src = a.q + (((size_t)(ok ? tt : tok0) * L.Hq + (size_t)h * G + rr % G) * ROW) + j * 16;
-    cp_async16_zfill(sQ + pa_swz(rr, j), src, ok);
-  }
-  auto load_kv = [&](int jt) {
-    const uint32_t sK = smem_u32(smem + kPaK);
-    const uint32_t sV = smem_u32(smem + kPaV);
-    for (int i = tid; i < kPaSlots * 16; i += kPaThreads) {
-      const int rr = i >> 4, j = i & 15;
-      const int slot = jt * kPaSlots + rr;
-      const bool ok = slot < vis_hi;
-      const int page = ok ? ptab[slot / kPage] : 0;
-      const char* src = L.pages + (size_t)page * L.page_bytes + (size_t)(ok ? slot % kPage : 0) * ROW + j * 16;
-      cp_async16_zfill(sK + pa_swz(rr, j), src, ok);
-      cp_async16_zfill(sV + pa_swz(rr, j), src + (size_t)kPage * ROW, ok);
-    }
-  };
-  if (ntiles > 0) load_kv(0);
-  cp_async_commit();
 
   tc_fence_before();
   __syncthreads();
@@ -366,7 +389,7 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
     }
     // P V done: O holds this tile, the K (P) and V buffers are free
     wait_bar(1, jt & 1);
-    if (jt + 1 < ntiles) load_kv(jt + 1);
+    if (jt + 1 < ntiles) load_kv(jt + 1, vis_hi);
     cp_async_commit();
   }
   cp_async_wait<0>();
@@ -396,13 +419,24 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
     const bool isv = tid >= D;
     unsigned char* buf = isv ? rv : rk;
     float acc = s_op[0] ? 0.f : carry[(isv ? D : 0) + col];
-    for (int i = 0; i < nrows; ++i) {
-      if (s_op[i]) acc = 0.f;
-      __nv_bfloat16* e = reinterpret_cast<__nv_bfloat16*>(buf + scr(i, col));
-      float x = __bfloat162float(*e);
-      if (!isv && col == 0) x = 0.f;  // k[0] <- 0 (Algorithm 1)
-      acc = fmaf(s_om[i], x, acc);
-      *e = __float2bfloat16_rn(acc * s_rz[i]);  // this token's running mean
+    const bool zero = !isv && col == 0;  // k[0] <- 0 (Algorithm 1)
+#pragma unroll 1
+    for (int i0 = 0; i0 < nrows; i0 += 8) {
+      float x[8];  // eight rows' loads in flight, then the serial sums
+#pragma unroll
+      for (int u = 0; u < 8; ++u)
+        x[u] = (i0 + u < nrows) ? __bfloat162float(*reinterpret_cast<const __nv_bfloat16*>(buf + scr(i0 + u, col)))
+                                : 0.f;
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const int i = i0 + u;
+        if (i < nrows) {
+          if (s_op[i]) acc = 0.f;
+          acc = fmaf(s_om[i], zero ? 0.f : x[u], acc);
+          // this token's running mean
+          *reinterpret_cast<__nv_bfloat16*>(buf + scr(i, col)) = __float2bfloat16_rn(acc * s_rz[i]);
+        }
+      }
     }
   }
   __syncthreads();
