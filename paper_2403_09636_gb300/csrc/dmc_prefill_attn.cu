@@ -34,8 +34,8 @@ constexpr int kPaSlots = 128;    // slots per K/V tile (N of S, K of P V)
 constexpr int kPaThreads = 256;  // two threads per query row, each half of its columns
 constexpr int kPaD = 128;        // head_dim handled by this kernel
 constexpr int kPaTileBytes = kPaRows * kPaD * 2;  // 32 KB: [128 rows][256 B]
-// dynamic shared memory: Q | K (then P) | V | misc, 100 KB: two CTAs per SM
-constexpr int kPaQ = 0, kPaK = kPaTileBytes, kPaV = 2 * kPaTileBytes, kPaP = kPaK;
+// dynamic shared memory: Q | K | V | misc, 100 KB: two CTAs per SM (P lives in TMEM)
+constexpr int kPaQ = 0, kPaK = kPaTileBytes, kPaV = 2 * kPaTileBytes;
 constexpr int kPaMisc = 3 * kPaTileBytes;
 constexpr int kPaSmem = kPaMisc + 4096;
 
@@ -77,6 +77,22 @@ __device__ __forceinline__ void pa_mma(uint32_t d_tmem, uint64_t a, uint64_t b, 
       "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
       "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
       "l"(a), "l"(b), "r"(idesc), "r"(acc ? 1 : 0));
+}
+
+// the same with A (M x K, bf16 pairs packed in 32-bit columns) read from tensor memory
+__device__ __forceinline__ void pa_mma_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b, uint32_t idesc,
+                                          bool acc) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(b), "r"(idesc), "r"(acc ? 1 : 0));
+}
+
+// 2^x by the SFU (ex2.approx, flushing subnormal results to zero)
+__device__ __forceinline__ float pa_ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
 }
 
 __device__ __forceinline__ void pa_commit(uint32_t bar) {
@@ -182,20 +198,23 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
     const char* src = a.q + (((size_t)(ok ? tt : tok0) * L.Hq + (size_t)h * G + rr % G) * ROW) + j * 16;
     cp_async16_zfill(sQ + pa_swz(rr, j), src, ok);
   }
-  auto load_kv = [&](int jt, int hi) {
-    const uint32_t sK = smem_u32(smem + kPaK);
-    const uint32_t sV = smem_u32(smem + kPaV);
+  // K (which = 0) or V (which = 1) rows of slot tile jt, slots below hi
+  auto load_tile = [&](int which, int jt, int hi) {
+    const uint32_t dst = smem_u32(smem + (which ? kPaV : kPaK));
     for (int i = tid; i < kPaSlots * 16; i += kPaThreads) {
       const int rr = i >> 4, j = i & 15;
       const int slot = jt * kPaSlots + rr;
       const bool ok = slot < hi;
       const int page = ok ? ptab[slot / kPage] : 0;
-      const char* src = L.pages + (size_t)page * L.page_bytes + (size_t)(ok ? slot % kPage : 0) * ROW + j * 16;
-      cp_async16_zfill(sK + pa_swz(rr, j), src, ok);
-      cp_async16_zfill(sV + pa_swz(rr, j), src + (size_t)kPage * ROW, ok);
+      const char* src = L.pages + (size_t)page * L.page_bytes +
+                        (size_t)(ok ? slot % kPage : 0) * ROW + (size_t)which * kPage * ROW + j * 16;
+      cp_async16_zfill(dst + pa_swz(rr, j), src, ok);
     }
   };
-  load_kv(0, min(kPaSlots, len_final));
+  // copy groups, oldest first: Q + K0, V0, then per tile K(j + 1) and V(j + 1)
+  load_tile(0, 0, min(kPaSlots, len_final));
+  cp_async_commit();
+  load_tile(1, 0, min(kPaSlots, len_final));
   cp_async_commit();
 
   // ---- per-token decisions, omega, slot counts and 1 / z of the chunk up to
@@ -303,9 +322,15 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
     }
   };
 
+  // Per slot tile j, with P kept in tensor memory so that the K buffer frees
+  // as soon as S is computed:
+  //   K(j) landed -> S = Q K^T -> K(j + 1) starts -> softmax, P (bf16) over
+  //   this thread's own S columns -> V(j) landed -> O += P V -> V(j + 1) starts
+  // The copy groups stay in step (one, possibly empty, per K and per V slot),
+  // so "all but the newest group" always means the tile needed next.
   float m = -INFINITY, l = 0.f;  // l: this thread's half of the row sum
   for (int jt = 0; jt < ntiles; ++jt) {
-    cp_async_wait<0>();  // Q and tile jt have landed (this thread's copies)
+    cp_async_wait<1>();  // Q and K(jt) have landed (this thread's copies)
     fence_async_smem();
     __syncthreads();
     if (tid == 0) {
@@ -318,78 +343,102 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
       }
       pa_commit(smem_u32(&bars[0]));
     }
-    wait_bar(0, jt & 1);  // S is in TMEM; the K buffer is free for P
+    wait_bar(0, jt & 1);  // S is in TMEM and the K buffer is free
     tc_fence_after();
-    // ---- online softmax: this thread's half of the row
+    if (jt + 1 < ntiles) load_tile(0, jt + 1, vis_hi);
+    cp_async_commit();
+    // ---- online softmax: this thread's half of the row. The running maximum m
+    // moves only when a tile's row maximum exceeds it by more than 8 (P then
+    // stays below 2^8; O and l are rescaled only on a move), in the log2 domain.
     const int vis_row = min(max(nvis - jt * kPaSlots, 0), kPaSlots);  // visible columns of the row
     const int vis_me = min(max(vis_row - (int)col0, 0), HALF);         // ... in this half
     const int vis_warp = __reduce_max_sync(0xffffffffu, vis_me);       // TMEM loads are warp-wide
-    float mx = -INFINITY;
+    const bool full = __all_sync(0xffffffffu, vis_me == HALF);         // no mask in this warp
+    float mx = -INFINITY;  // of the raw scores
     for (int c0 = 0; c0 < vis_warp; c0 += 32) {
       float f[32];
       pa_ld32(tS + lane_base + col0 + c0, f);
+      if (full) {
 #pragma unroll
-      for (int i = 0; i < 32; ++i)
-        if (c0 + i < vis_me) mx = fmaxf(mx, f[i] * qscale);
+        for (int i = 0; i < 32; ++i) mx = fmaxf(mx, f[i]);
+      } else {
+#pragma unroll
+        for (int i = 0; i < 32; ++i)
+          if (c0 + i < vis_me) mx = fmaxf(mx, f[i]);
+      }
     }
-    s_x[hf * kPaRows + r] = mx;
+    s_x[hf * kPaRows + r] = mx * qscale;  // qscale > 0
     __syncthreads();
-    const float mn = fmaxf(m, fmaxf(mx, s_x[(hf ^ 1) * kPaRows + r]));
+    const float mt = fmaxf(mx * qscale, s_x[(hf ^ 1) * kPaRows + r]);  // the tile's row maximum
+    const bool grow = mt > m + 8.f;  // false while the row has seen nothing
+    const float mn = grow ? mt : m;
+    const float nmn = -mn;
     float sum = 0.f;
-    unsigned char* sP = smem + kPaP;
+    uint32_t pk[HALF / 2];  // P of this half, bf16 pairs
+#pragma unroll
     for (int c0 = 0; c0 < HALF; c0 += 32) {
       float f[32];
       if (c0 < vis_warp) {
         pa_ld32(tS + lane_base + col0 + c0, f);
+        if (full) {
+#pragma unroll
+          for (int i = 0; i < 32; ++i) f[i] = pa_ex2(fmaf(f[i], qscale, nmn));
+        } else {
+#pragma unroll
+          for (int i = 0; i < 32; ++i) f[i] = (c0 + i < vis_me) ? pa_ex2(fmaf(f[i], qscale, nmn)) : 0.f;
+        }
       } else {
 #pragma unroll
         for (int i = 0; i < 32; ++i) f[i] = 0.f;
       }
 #pragma unroll
-      for (int i = 0; i < 32; ++i) {
-        const float p = (c0 + i < vis_me) ? exp2f(f[i] * qscale - mn) : 0.f;
-        f[i] = p;
-        sum += p;
-      }
+      for (int i = 0; i < 32; ++i) sum += f[i];
 #pragma unroll
-      for (int q4 = 0; q4 < 4; ++q4)
-        *reinterpret_cast<uint4*>(sP + pa_swz(r, ((col0 + c0) >> 3) + q4)) =
-            Chunk<__nv_bfloat16>::pack(f + q4 * 8);
+      for (int i = 0; i < 16; ++i) pk[c0 / 2 + i] = Chunk<__nv_bfloat16>::pack2(f[2 * i], f[2 * i + 1]);
     }
-    const float corr = (m == -INFINITY) ? 0.f : exp2f(m - mn);
+    // P over the first half of this thread's own S columns: slots col0 + 2i,
+    // col0 + 2i + 1 in column col0 + i (the other half's thread writes its own)
+    {
+      float pf[32];
+#pragma unroll
+      for (int i = 0; i < 32; ++i) pf[i] = __uint_as_float(pk[i]);
+      pa_st32(tS + lane_base + col0, pf);
+    }
+    // a move of the maximum rescales l and this half of O (rows that saw
+    // nothing yet hold zeros)
+    const bool resc = grow && m != -INFINITY;
+    const float corr = resc ? pa_ex2(m - mn) : 1.f;
     l = l * corr + sum;
-    // rescale this half of O rows whose maximum moved (rows that saw nothing
-    // yet hold zeros)
-    const bool resc = jt > 0 && corr != 1.f;
     if (__any_sync(0xffffffffu, resc)) {
-      const float cr = resc ? corr : 1.f;
       for (int c0 = 0; c0 < HALF; c0 += 32) {
         float f[32];
         pa_ld32(tO + lane_base + col0 + c0, f);
 #pragma unroll
-        for (int i = 0; i < 32; ++i) f[i] *= cr;
+        for (int i = 0; i < 32; ++i) f[i] *= corr;
         pa_st32(tO + lane_base + col0 + c0, f);
       }
-      asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
     }
-    if (mn != -INFINITY) m = mn;
+    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+    m = mn;
+    cp_async_wait<1>();  // V(jt) has landed (K(jt + 1) may still be on its way)
     fence_async_smem();
     tc_fence_before();
     __syncthreads();
     if (tid == 0) {
       tc_fence_after();
-      const uint32_t pA = smem_u32(smem + kPaP), vB = smem_u32(smem + kPaV);
+      const uint32_t vB = smem_u32(smem + kPaV);
 #pragma unroll
       for (int kk = 0; kk < kPaSlots / 16; ++kk) {
-        const uint32_t aoff = (kk >> 2) * (kPaRows * 128) + (kk & 3) * 32;
-        pa_mma(tO, pa_desc(pA + aoff, 16, 1024), pa_desc(vB + kk * 2048, kPaRows * 128, 1024),
-               pa_idesc(true), jt > 0 || kk > 0);
+        // slots 16 kk ... from half kk / 4 of the row, 8 packed columns per step
+        const uint32_t aT = tS + (uint32_t)((kk >> 2) * HALF + (kk & 3) * 8);
+        pa_mma_ts(tO, aT, pa_desc(vB + kk * 2048, kPaRows * 128, 1024), pa_idesc(true), jt > 0 || kk > 0);
       }
       pa_commit(smem_u32(&bars[1]));
     }
-    // P V done: O holds this tile, the K (P) and V buffers are free
+    // P V done: O holds this tile, S (P) and the V buffer are free
     wait_bar(1, jt & 1);
-    if (jt + 1 < ntiles) load_kv(jt + 1, vis_hi);
+    tc_fence_after();
+    if (jt + 1 < ntiles) load_tile(1, jt + 1, vis_hi);
     cp_async_commit();
   }
   cp_async_wait<0>();
