@@ -55,6 +55,8 @@ def parse():
                     help="override the workload's decode steps (not for reported numbers)")
     ap.add_argument("--layers", type=int, default=None,
                     help="override the workload's layer count (small ncu cases, not for reported numbers)")
+    ap.add_argument("--batch", type=int, default=None,
+                    help="override the workload's batch (small ncu cases, not for reported numbers)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -253,6 +255,8 @@ def run_ours(args, rank, world, dist):
     wl = S.WORKLOADS[args.workload]
     if args.layers is not None:
         wl = S.shrink(wl, num_layers=args.layers)
+    if args.batch is not None:
+        wl = S.shrink(wl, batch=args.batch)
     steps_dec = wl.decode_steps if args.decode_steps is None else args.decode_steps
     Lr, Bt, Hq, Hk, D = wl.num_layers, wl.batch, wl.num_q_heads, wl.num_kv_heads, wl.head_dim
     dt = wl.torch_dtype

@@ -149,7 +149,7 @@ __device__ __forceinline__ float* carry_at(const PrefillArgs& a, int t0, int cs,
 }
 
 template <typename T, int D>
-__device__ __forceinline__ void scan_segment(const PrefillArgs& a, int h, int bh, int tb, int te,
+__device__ __noinline__ void scan_segment(const PrefillArgs& a, int h, int bh, int tb, int te,
                                              int slot, bool merge_old, int t0, int s, int t1) {
   using CK = Chunk<T>;
   constexpr int ROW = D * (int)sizeof(T);
@@ -287,11 +287,12 @@ __device__ __forceinline__ void scan_segment(const PrefillArgs& a, int h, int bh
   // the lr == 0 lane holds z; every lane needs it for the quotient
   zs = __shfl_sync(0xffffffffu, zs, lane - lr);
   if (sub != 0) return;
+  const float iz = 1.f / zs;
   float kn[EPC], vn[EPC];
 #pragma unroll
   for (int e = 0; e < EPC; ++e) {
-    kn[e] = ak[e] / zs;
-    vn[e] = av[e] / zs;
+    kn[e] = ak[e] * iz;
+    vn[e] = av[e] * iz;
   }
   if (lr == 0) kn[0] = 0.f;
   *reinterpret_cast<uint4*>(kdst) = CK::pack(kn);
