@@ -583,11 +583,12 @@ def run_e2e(args, wl, cache, prompts, qd, kd, vd, outs, steps_dec, dev, stream, 
     each step copies every layer's prompt (one layer's pinned prompt reused for
     all layers) and every decode step's q/k/v (a pinned ring of `ring`
     distinct steps reused cyclically), and reads every decode output back into
-    a pinned ring. The copies run on two copy streams, as a server prefetches
-    its next inputs: the next step's prompts while this step decodes, the next
-    decode steps' q/k/v two steps ahead, each step's outputs as soon as they
-    are written; events order every copy against the kernels that use its
-    buffer."""
+    a pinned ring. The copies run on one copy stream, as a server prefetches
+    its next inputs: each step's outputs as soon as they are written, the
+    decode inputs two steps ahead (double-buffered), and the next step's
+    prompts in token slices, a few after each decode step's input copy, so
+    that no input copy waits behind a whole prompt; events order every copy
+    against the kernels that use its buffer."""
     import torch
 
     Lr = wl.num_layers
@@ -617,23 +618,32 @@ def run_e2e(args, wl, cache, prompts, qd, kd, vd, outs, steps_dec, dev, stream, 
         gv[0].numel() * gv[0].element_size())
     d2h = steps_dec * outs.numel() * outs.element_size()
 
-    cs_p = torch.cuda.Stream(dev)   # prompt copies
-    cs_io = torch.cuda.Stream(dev)  # decode inputs and outputs
+    cs_io = torch.cuda.Stream(dev)  # every copy, in the order the kernels need them
     ev = lambda: torch.cuda.Event()
     ev_pr = [ev() for _ in range(Lr)]   # prompt of layer l landed
-    ev_pf = [ev() for _ in range(Lr)]   # prefill of layer l done with its buffer
+    ev_pf = ev()                        # this step's prefill is done with the prompt buffers
     ev_in = [ev() for _ in range(2)]    # decode inputs of buffer b landed
     ev_done = [ev() for _ in range(2)]  # decodes of buffer b done (inputs free, outputs ready)
     ev_d2h = [ev() for _ in range(2)]   # outputs of buffer b read back
+    # the next step's prompts go in NC token slices, a few after each decode
+    # step's input copy, so that no input copy waits behind a whole prompt
+    CPL = 16                            # slices per layer
+    NC = Lr * CPL
+    bounds = [tot * j // CPL for j in range(CPL + 1)]
 
-    def copy_prompts():
-        with torch.cuda.stream(cs_p):
-            for l in range(Lr):
-                cs_p.wait_event(ev_pf[l])
-                dq0[l].copy_(hq0, non_blocking=True)
-                dk[l].copy_(hk, non_blocking=True)
-                dv[l].copy_(hv, non_blocking=True)
-                ev_pr[l].record(cs_p)
+    def copy_prompt_slice(k):  # on cs_io
+        l, j = divmod(k, CPL)
+        a, b = bounds[j], bounds[j + 1]
+        dq0[l][a:b].copy_(hq0[a:b], non_blocking=True)
+        dk[l][a:b].copy_(hk[a:b], non_blocking=True)
+        dv[l][a:b].copy_(hv[a:b], non_blocking=True)
+        if j == CPL - 1:
+            ev_pr[l].record(cs_io)
+
+    def copy_prompts():  # all at once (the first step's)
+        with torch.cuda.stream(cs_io):
+            for k in range(NC):
+                copy_prompt_slice(k)
 
     def copy_inputs(t, b):
         with torch.cuda.stream(cs_io):
@@ -645,7 +655,6 @@ def run_e2e(args, wl, cache, prompts, qd, kd, vd, outs, steps_dec, dev, stream, 
 
     def run(nsteps):
         # the first step's prompts and first two decode steps' inputs
-        cs_p.wait_stream(stream)
         cs_io.wait_stream(stream)
         copy_prompts()
         copy_inputs(0, 0)
@@ -657,9 +666,11 @@ def run_e2e(args, wl, cache, prompts, qd, kd, vd, outs, steps_dec, dev, stream, 
                 rc |= L_.dmc_prefill_compress(h, l, 0, ns, dq0[l].data_ptr(), dq0[l].stride(0),
                                               dq0[l].stride(1), dk[l].data_ptr(), dv[l].data_ptr(),
                                               cu.data_ptr(), tot, mx, sh)
-                ev_pf[l].record(stream)
-            if i + 1 < nsteps:
-                copy_prompts()  # the next step's, while this one decodes
+            ev_pf.record(stream)
+            nxt = i + 1 < nsteps  # the next step's prompts stream during this step's decode
+            if nxt:
+                with torch.cuda.stream(cs_io):
+                    cs_io.wait_event(ev_pf)
             for t in range(steps_dec):
                 b = t & 1
                 stream.wait_event(ev_in[b])
@@ -676,9 +687,12 @@ def run_e2e(args, wl, cache, prompts, qd, kd, vd, outs, steps_dec, dev, stream, 
                 if not last:
                     # two steps ahead (at the end of a step, the next step's first two)
                     copy_inputs((t + 2) % steps_dec, b)
+                if nxt:
+                    with torch.cuda.stream(cs_io):
+                        for k in range(t * NC // steps_dec, (t + 1) * NC // steps_dec):
+                            copy_prompt_slice(k)
             if rc:
                 raise RuntimeError(f"launch failed: {rc}")
-        stream.wait_stream(cs_p)
         stream.wait_stream(cs_io)
 
     run(max(1, args.warmup))
@@ -696,8 +710,8 @@ def run_e2e(args, wl, cache, prompts, qd, kd, vd, outs, steps_dec, dev, stream, 
             "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
             "note": f"pinned host inputs: one layer's prompt reused for all {Lr} layers, a ring of "
                     f"{ring} decode steps reused cyclically; every attention output is read back into a "
-                    f"pinned ring of {ring} steps; copies on two side streams overlap the kernels "
-                    "(next step's prompts during this step's decode, decode inputs two steps ahead)"}
+                    f"pinned ring of {ring} steps; copies on a side stream overlap the kernels "
+                    "(decode inputs two steps ahead; the next step's prompts in slices between them)"}
 
 
 def main():
