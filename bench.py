@@ -229,12 +229,21 @@ def oracle_rate(wl, seconds, decode_steps, threads=None):
     instances = wl.num_layers * wl.batch * wl.num_kv_heads
     job_s = per_instance * instances
     rate = wl.batch * decode_steps / job_s
+    # the same on one thread, over the first few instances
+    n1 = min(16, len(order))
+    one = [instance(*order[i]) for i in range(n1)]
+    t0 = time.perf_counter()
+    cref.run_heads(one, threads=1, want_out=True, want_prompt_slots=False)
+    spent1 = time.perf_counter() - t0
     rec = {"value": rate, "unit": "tokens/s", "cores": threads, "kind": "oracle",
            "sample": (f"C fp64 oracle (oracle/dmc_ref.c), {done} (layer 0, seq, kv-head) instances "
                       f"of {wl.name}, each {int(lens.mean())} prompt + {decode_steps} decode tokens, "
                       f"{spent:.1f} s on {threads} threads; extrapolated linearly to "
                       f"{instances} instances ({wl.num_layers} layers)"),
-           "seconds": spent}
+           "seconds": spent,
+           "single_thread": {"value": wl.batch * decode_steps / (spent1 / n1 * instances),
+                             "unit": "tokens/s", "cores": 1,
+                             "sample": f"{n1} instances, {spent1:.2f} s on one thread, extrapolated alike"}}
     return rate, rec
 
 
