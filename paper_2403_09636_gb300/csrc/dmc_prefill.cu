@@ -13,14 +13,17 @@
 //  scan: one block per (128-token chunk, KV head, sequence). The block owns the
 //        segments that open inside its chunk (and chunk 0 also owns the tokens
 //        that continue the head's existing last slot); a segment that runs past
-//        the chunk end is followed to its end, so each k/v row is read once.
-//        Warps take segments round-robin; lanes split a row into 16-byte pieces
-//        and accumulate sum(omega k), sum(omega v), sum(omega) in fp32; the slot
-//        is the quotient, rounded once to the cache dtype. When asked for
+//        the chunk end is followed to its end. Lanes split a row into 16-byte
+//        pieces and accumulate sum(omega k), sum(omega v), sum(omega) in fp32;
+//        the slot is the quotient, rounded once to the cache dtype. Exact
+//        compression walks the chunk's tokens in row groups (see the kernel);
+//        window grouping gives each segment to one warp. When asked for
 //        (prompt attention), the block also records, at every chunk start a
 //        segment runs across, the segment's sums up to that point (the
 //        "carry"), so that each chunk can rebuild the running state of its
 //        tokens without reading back to the segment's start.
+//  ring: window grouping only, after the scan: stores each head's open
+//        segment's last W - 1 tokens and its length.
 #include "dmc_internal.cuh"
 
 namespace dmc {
@@ -148,9 +151,14 @@ __device__ __forceinline__ float* carry_at(const PrefillArgs& a, int t0, int cs,
   return a.carry + ((size_t)chunk_id(t0, (cs - t0) / kPrefillChunk, s) * a.lay.Hkv + h) * (2 * D + 1);
 }
 
+// Window grouping: one warp sums segment [tb, te) into `slot`, counting only
+// its last W tokens; the head's open segment keeps its last W - 1 tokens in
+// the ring (token p of the segment at entry p % W) and its length in seglen,
+// and a prompt that continues it (merge_old) takes the continued segment's
+// tokens still inside the window from there.
 template <typename T, int D>
-__device__ __noinline__ void scan_segment(const PrefillArgs& a, int h, int bh, int tb, int te,
-                                             int slot, bool merge_old, int t0, int s, int t1) {
+__device__ __noinline__ void scan_window_segment(const PrefillArgs& a, int h, int bh, int tb,
+                                                 int te, int slot, bool merge_old) {
   using CK = Chunk<T>;
   constexpr int ROW = D * (int)sizeof(T);
   constexpr int LPR = ROW / 16;  // lanes per row
@@ -166,114 +174,49 @@ __device__ __noinline__ void scan_segment(const PrefillArgs& a, int h, int bh, i
   char* kdst = L.pages + (size_t)page * L.page_bytes + (size_t)(slot % kPage) * ROW + lr * 16;
   char* vdst = kdst + (size_t)kPage * ROW;
   float* zp = L.z + (size_t)page * kPage + slot % kPage;
-  // Window grouping (W > 0): the slot is the mean of the segment's last W
-  // tokens only; the head's open segment keeps its last W - 1 tokens in the
-  // ring (token p of the segment at entry p % W) and its length in seglen.
   const int W = L.window;
-  int* seglen = nullptr;
-  char* ring = nullptr;
-  float* ring_w = nullptr;
-  int n_old = 0;  // tokens of the continued segment before this prompt
-  if (W > 0) {
-    const int parity = *reinterpret_cast<const volatile int*>(&L.ctl[a.layer * 4]);
-    seglen = L.seglen + ((size_t)a.layer * 2 + parity) * L.NH + bh;
-    ring = L.ring + ((size_t)a.layer * L.NH + bh) * W * 2 * ROW;
-    ring_w = L.ring_w + ((size_t)a.layer * L.NH + bh) * W;
-    if (merge_old) n_old = *seglen;
-  }
-  const int sb = W > 0 ? max(tb, te - W) : tb;  // first token the slot counts
+  const int parity = *reinterpret_cast<const volatile int*>(&L.ctl[a.layer * 4]);
+  const char* ring = L.ring + ((size_t)a.layer * L.NH + bh) * W * 2 * ROW;
+  const float* ring_w = L.ring_w + ((size_t)a.layer * L.NH + bh) * W;
   if (merge_old && sub == 0) {
-    if (W == 0) {
-      // the prompt continues the head's last slot: its K z_old, V z_old and
-      // z_old join the sums (one copy, in the first row group's lanes)
+    // the continued segment's tokens still inside the window, from the ring
+    const int n_old = L.seglen[((size_t)a.layer * 2 + parity) * L.NH + bh];
+    const int m = min(n_old, max(0, W - (te - tb)));
+    for (int e = 0; e < m; ++e) {
+      const int pos = (n_old - 1 - e) % W;
       float ko[EPC], vo[EPC];
-      CK::unpack(*reinterpret_cast<const uint4*>(kdst), ko);
-      CK::unpack(*reinterpret_cast<const uint4*>(vdst), vo);
-      const float zo = *zp;
+      CK::unpack(*reinterpret_cast<const uint4*>(ring + (size_t)pos * 2 * ROW + lr * 16), ko);
+      CK::unpack(*reinterpret_cast<const uint4*>(ring + (size_t)pos * 2 * ROW + ROW + lr * 16), vo);
+      const float w = ring_w[pos];
 #pragma unroll
-      for (int e = 0; e < EPC; ++e) {
-        ak[e] = ko[e] * zo;
-        av[e] = vo[e] * zo;
+      for (int e2 = 0; e2 < EPC; ++e2) {
+        ak[e2] = fmaf(w, ko[e2], ak[e2]);
+        av[e2] = fmaf(w, vo[e2], av[e2]);
       }
-      zs = lr == 0 ? zo : 0.f;
-    } else {
-      // the continued segment's tokens still inside the window, from the ring
-      const int m = min(n_old, max(0, W - (te - tb)));
-      for (int e = 0; e < m; ++e) {
-        const int pos = (n_old - 1 - e) % W;
-        float ko[EPC], vo[EPC];
-        CK::unpack(*reinterpret_cast<const uint4*>(ring + (size_t)pos * 2 * ROW + lr * 16), ko);
-        CK::unpack(*reinterpret_cast<const uint4*>(ring + (size_t)pos * 2 * ROW + ROW + lr * 16), vo);
-        const float w = ring_w[pos];
-#pragma unroll
-        for (int e2 = 0; e2 < EPC; ++e2) {
-          ak[e2] = fmaf(w, ko[e2], ak[e2]);
-          av[e2] = fmaf(w, vo[e2], av[e2]);
-        }
-        if (lr == 0) zs += w;
-      }
+      if (lr == 0) zs += w;
     }
   }
-  // Writes the sums so far (all row groups together) as the carry of the chunk
-  // starting at token cs.
-  auto put_carry = [&](int cs) {
-    float sk[EPC], sv[EPC];
-    float sz = zs;
-#pragma unroll
-    for (int e = 0; e < EPC; ++e) { sk[e] = ak[e]; sv[e] = av[e]; }
-#pragma unroll
-    for (int off = LPR; off < 32; off <<= 1) {
-#pragma unroll
-      for (int e = 0; e < EPC; ++e) {
-        sk[e] += __shfl_xor_sync(0xffffffffu, sk[e], off);
-        sv[e] += __shfl_xor_sync(0xffffffffu, sv[e], off);
-      }
-      sz += __shfl_xor_sync(0xffffffffu, sz, off);
-    }
-    if (sub == 0) {
-      float* cp = carry_at(a, t0, cs, s, h, D);
-#pragma unroll
-      for (int e = 0; e < EPC; ++e) {
-        cp[lr * EPC + e] = sk[e];
-        cp[D + lr * EPC + e] = sv[e];
-      }
-      if (lr == 0) cp[2 * D] = sz;
-    }
-  };
-  const bool carry = a.carry != nullptr;
-  if (carry && merge_old) put_carry(t0);  // the state the prompt's first token continues
   const size_t hrow = (size_t)L.Hkv * ROW;
   const char* kb = a.k + (size_t)h * ROW + lr * 16;
   const char* vb = a.v + (size_t)h * ROW + lr * 16;
-  // the segment in pieces that end at chunk starts (only split when carries are asked for)
-  int pb = sb;
-  while (pb < te) {
-    int pe = te;
-    if (carry) {
-      const int next_chunk = t0 + ((pb - t0) / kPrefillChunk + 1) * kPrefillChunk;
-      pe = min(te, next_chunk);
-    }
 #pragma unroll 2
-    for (int t = pb + sub; t < pe; t += RPI) {
-      const uint4 kr = __ldg(reinterpret_cast<const uint4*>(kb + (size_t)t * hrow));
-      const uint4 vr = __ldg(reinterpret_cast<const uint4*>(vb + (size_t)t * hrow));
-      float y = 0.f;
-      for (int g = 0; g < L.G; ++g)
-        y += Elt<T>::to_f(qq[(size_t)t * a.q_tok + (size_t)(h * L.G + g) * a.q_head]);
-      const float w = sigmoidf_(y / (float)L.G);  // omega = sigmoid(q[0]) (group mean for GQA)
-      float kf[EPC], vf[EPC];
-      CK::unpack(kr, kf);
-      CK::unpack(vr, vf);
-      if (lr == 0) kf[0] = 0.f;  // k[0] <- 0 (Algorithm 1)
+  for (int t = max(tb, te - W) + sub; t < te; t += RPI) {  // the segment's last W tokens
+    const uint4 kr = __ldg(reinterpret_cast<const uint4*>(kb + (size_t)t * hrow));
+    const uint4 vr = __ldg(reinterpret_cast<const uint4*>(vb + (size_t)t * hrow));
+    float y = 0.f;
+    for (int g = 0; g < L.G; ++g)
+      y += Elt<T>::to_f(qq[(size_t)t * a.q_tok + (size_t)(h * L.G + g) * a.q_head]);
+    const float w = sigmoidf_(y / (float)L.G);  // omega = sigmoid(q[0]) (group mean for GQA)
+    float kf[EPC], vf[EPC];
+    CK::unpack(kr, kf);
+    CK::unpack(vr, vf);
+    if (lr == 0) kf[0] = 0.f;  // k[0] <- 0 (Algorithm 1)
 #pragma unroll
-      for (int e = 0; e < EPC; ++e) {
-        ak[e] = fmaf(w, kf[e], ak[e]);
-        av[e] = fmaf(w, vf[e], av[e]);
-      }
-      zs += w;
+    for (int e = 0; e < EPC; ++e) {
+      ak[e] = fmaf(w, kf[e], ak[e]);
+      av[e] = fmaf(w, vf[e], av[e]);
     }
-    if (pe < te) put_carry(pe);  // the segment runs across the chunk starting at pe
-    pb = pe;
+    zs += w;
   }
 #pragma unroll
   for (int off = LPR; off < 32; off <<= 1) {
@@ -682,12 +625,12 @@ __global__ void __launch_bounds__(kScanThreads) dmc_prefill_scan_window_kernel(c
   for (int it = warp; it < items; it += kScanThreads / 32) {
     if (pre && it == 0) {
       const int te = nstart > 0 ? starts[0] : next;
-      scan_segment<T, D>(a, h, bh, t0, te, base - 1, true, t0, s, t1);
+      scan_window_segment<T, D>(a, h, bh, t0, te, base - 1, true);
     } else {
       const int j = it - (pre ? 1 : 0);
       const int tb = starts[j];
       const int te = (j + 1 < nstart) ? starts[j + 1] : next;
-      scan_segment<T, D>(a, h, bh, tb, te, base + j, false, t0, s, t1);
+      scan_window_segment<T, D>(a, h, bh, tb, te, base + j, false);
     }
   }
 }
