@@ -61,3 +61,43 @@ def test_graph_replay_matches_eager(cuda_dev, wl):
         assert torch.equal(graphed.lengths(layer), eager.lengths(layer))
     assert graphed.status()[:2] == (0, 0)
     assert eager.status()[:2] == (0, 0)
+
+
+@pytest.mark.parametrize("wl", CASES[:2], ids=lambda w: w.name)
+def test_graph_prompt_and_decode_replay_matches_eager(cuda_dev, wl):
+    """A whole step in one graph: reset, prompt attention (plan, the scan
+    launched as a programmatic dependent, the attention kernel) for every
+    layer, then one decode step of every layer. Each replay must give exactly
+    the eager step's attention outputs and slot counts (page ids may differ:
+    heads take pages from the pool in a racy order)."""
+    p = S.append_prob(wl)
+    eager, graphed = H.cache_for(wl, cuda_dev), H.cache_for(wl, cuda_dev)
+    prompts = [S.gen_prompt(wl, layer, cuda_dev, p=p, full_q=True) for layer in range(wl.num_layers)]
+    dec = [S.gen_decode(wl, layer, 0, cuda_dev, p=p) for layer in range(wl.num_layers)]
+    pa_g = [torch.empty_like(pr["q"]) for pr in prompts]
+    o_g = [torch.empty_like(x["q"]) for x in dec]
+
+    def step(cache, pa_out, dec_out):
+        cache.reset()
+        for layer, pr in enumerate(prompts):
+            cache.prefill_attention(layer, pr["q"], pr["k"], pr["v"], pr["cu_seqlens"], pr["max_seqlen"],
+                                    pa_out[layer])
+        for layer, x in enumerate(dec):
+            cache.decode(layer, x["q"], x["k"], x["v"], dec_out[layer])
+
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        step(graphed, pa_g, o_g)
+    for rep in range(2):
+        pa_e = [torch.empty_like(pr["q"]) for pr in prompts]
+        o_e = [torch.empty_like(x["q"]) for x in dec]
+        step(eager, pa_e, o_e)
+        g.replay()
+        torch.cuda.synchronize()
+        for layer in range(wl.num_layers):
+            assert torch.equal(pa_g[layer], pa_e[layer]), (rep, layer)
+            assert torch.equal(o_g[layer], o_e[layer]), (rep, layer)
+            assert torch.equal(graphed.lengths(layer), eager.lengths(layer)), (rep, layer)
+        assert graphed.status()[:2] == (0, 0)
+        assert eager.status()[:2] == (0, 0)
