@@ -134,8 +134,8 @@ dmc_status dmc_prefill_compress(dmc_cache_t cache, int32_t layer, int32_t first_
  * continues its last segment, so splitting a prompt over calls gives the same
  * outputs. The score is q[1:]^T k[1:] / sqrt(head_dim) (q[0] and k[0] are the
  * gates). Runs on the tcgen05 tensor cores: bf16 caches with head_dim 128 and
- * 1, 2, 4 or 8 query heads per KV head; other caches return
- * DMC_ERR_INVALID_ARG.
+ * 1, 2, 4 or 8 query heads per KV head, exact compression (window = 0); other
+ * caches return DMC_ERR_INVALID_ARG.
  *   q_dev:   [total_tokens, num_q_heads, head_dim], packed (q[., ., 0] also
  *            gives omega, as in dmc_prefill_compress);
  *   k_dev, v_dev: [total_tokens, num_kv_heads, head_dim], sequences packed;
