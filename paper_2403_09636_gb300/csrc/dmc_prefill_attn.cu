@@ -34,10 +34,10 @@ constexpr int kPaSlots = 128;    // slots per K/V tile (N of S, K of P V)
 constexpr int kPaThreads = 256;  // two threads per query row, each half of its columns
 constexpr int kPaD = 128;        // head_dim handled by this kernel
 constexpr int kPaTileBytes = kPaRows * kPaD * 2;  // 32 KB: [128 rows][256 B]
-// dynamic shared memory: Q | K | V | misc, 100 KB: two CTAs per SM (P lives in TMEM)
+// dynamic shared memory: Q | K | V | misc, 104 KB: two CTAs per SM (P lives in TMEM)
 constexpr int kPaQ = 0, kPaK = kPaTileBytes, kPaV = 2 * kPaTileBytes;
 constexpr int kPaMisc = 3 * kPaTileBytes;
-constexpr int kPaSmem = kPaMisc + 4096;
+constexpr int kPaSmem = kPaMisc + 8192;
 
 struct PrefillAttnArgs {
   Layout lay;
@@ -169,6 +169,8 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
   int* s_wc = reinterpret_cast<int*>(smem + kPaMisc + 64 + 3712);      // [4] openings per warp
   int* s_wf = reinterpret_cast<int*>(smem + kPaMisc + 64 + 3728);      // [4] the warp has one
   float* s_wz = reinterpret_cast<float*>(smem + kPaMisc + 64 + 3744);  // [4] its last segment's omega sum
+  int* s_wm = reinterpret_cast<int*>(smem + kPaMisc + 64 + 3760);      // [4] its last opening token
+  int* s_seg = reinterpret_cast<int*>(smem + kPaMisc + 4096);          // [128] first token of the segment, or -1
 
   const int t0 = a.cu[s], t1 = a.cu[s + 1];
   if (!(t0 >= 0 && t0 <= t1 && t1 <= a.total_tokens && t1 - t0 <= a.max_seqlen)) return;
@@ -221,7 +223,7 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
   // the tile end. z after token i is the omega sum of i's segment so far: from
   // the segment's opening token, or from the carried sums when no token of the
   // chunk up to i opens a slot (a segmented prefix sum over the chunk).
-  int incl = 0, seg = 0;
+  int incl = 0, seg = 0, lastop = -1;
   float zs = 0.f;
   if (tid < kPrefillChunk) {
     const int tau = a0 + tid;
@@ -242,21 +244,25 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
     incl = op;
     seg = op;
     zs = om;
+    lastop = op ? tid : -1;  // the last opening token up to this one
 #pragma unroll
     for (int off = 1; off < 32; off <<= 1) {
       const int o = __shfl_up_sync(0xffffffffu, incl, off);
       const int so = __shfl_up_sync(0xffffffffu, seg, off);
       const float zo = __shfl_up_sync(0xffffffffu, zs, off);
+      const int lo = __shfl_up_sync(0xffffffffu, lastop, off);
       if (lane >= off) {
         incl += o;
         if (!seg) zs += zo;
         seg |= so;
+        lastop = max(lastop, lo);
       }
     }
     if (lane == 31) {
       s_wc[warp] = incl;
       s_wf[warp] = seg;
       s_wz[warp] = zs;
+      s_wm[warp] = lastop;
     }
   }
   if (tid == 0) {
@@ -275,6 +281,8 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
     int add = base;
     for (int w = 0; w < warp; ++w) add += s_wc[w];
     s_len[tid] = incl + add;  // slot count after token a0 + tid
+    for (int w = 0; w < warp; ++w) lastop = max(lastop, s_wm[w]);
+    s_seg[tid] = lastop;
     if (!seg) {
       // the segment runs in from earlier warps, or from before the chunk
       bool found = false;
@@ -443,94 +451,139 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
   }
   cp_async_wait<0>();
   tc_fence_after();
-  __syncthreads();  // every thread's reads of the K/V buffers are over
+  __syncthreads();  // every MMA and copy of the loop is over: the K and V buffers are free
 
-  // ---- the diagonal state of each token: segment sums from the chunk start
-  // Raw k, v rows of tokens [a0, tokN) go to the K / V buffers as 256-byte rows
-  // whose 16-byte chunks are XOR-swizzled by row (conflict-free row reads
-  // below); the running means then replace them in place.
-  auto scr = [&](int i, int col) { return i * ROW + ((((col >> 3) ^ (i & 15))) << 4) + (col & 7) * 2; };
-  unsigned char* rk = smem + kPaK;
-  unsigned char* rv = smem + kPaV;
+  // ---- the diagonal state as one more tile. When token i of the chunk
+  // attends, its own slot holds k~ = (c_k [no opening in the chunk up to i] +
+  // sum over j = lo..i of omega_j k_j) / z_i, lo being its segment's first
+  // token in the chunk (c_k: the carried sums), and v~ alike. Its score
+  // q . k~ and its share of O come from the chunk's raw rows:
+  // S_d = Q Kraw^T (with q[0] cleared: the gate is not a feature) summed with
+  // the weights omega_j / z_i, then O += P_d Vraw with
+  // P_d[j] = exp2(score - m) omega_j / z_i over the segment's columns.
   const int nrows = tokN - a0;
-  for (int i = tid; i < nrows * 16; i += kPaThreads) {
-    const int rr = i >> 4, j = i & 15;
-    const size_t src = ((size_t)(a0 + rr) * L.Hkv + h) * ROW + j * 16;
-    cp_async16(smem_u32(rk + scr(rr, j * 8)), a.k + src);
-    cp_async16(smem_u32(rv + scr(rr, j * 8)), a.v + src);
-  }
-  cp_async_commit();
-  cp_async_wait<0>();
-  __syncthreads();
-  // thread t runs column t % 128 of k (t < 128) or of v down the chunk
+  if (tid < kPaRows) *reinterpret_cast<__nv_bfloat16*>(smem + kPaQ + pa_swz(tid, 0)) = __float2bfloat16_rn(0.f);
   {
-    const int col = tid & (D - 1);
-    const bool isv = tid >= D;
-    unsigned char* buf = isv ? rv : rk;
-    float acc = s_op[0] ? 0.f : carry[(isv ? D : 0) + col];
-    const bool zero = !isv && col == 0;  // k[0] <- 0 (Algorithm 1)
-#pragma unroll 1
-    for (int i0 = 0; i0 < nrows; i0 += 8) {
-      float x[8];  // eight rows' loads in flight, then the serial sums
+    const uint32_t sK = smem_u32(smem + kPaK), sV = smem_u32(smem + kPaV);
+    for (int i = tid; i < kPaRows * 16; i += kPaThreads) {
+      const int rr = i >> 4, j = i & 15;
+      const bool ok = rr < nrows;
+      const size_t src = ((size_t)(a0 + (ok ? rr : 0)) * L.Hkv + h) * ROW + j * 16;
+      cp_async16_zfill(sK + pa_swz(rr, j), a.k + src, ok);
+      cp_async16_zfill(sV + pa_swz(rr, j), a.v + src, ok);
+    }
+    cp_async_commit();
+    cp_async_wait<0>();
+  }
+  fence_async_smem();
+  tc_fence_before();
+  __syncthreads();
+  if (tid == 0) {
+    tc_fence_after();
+    const uint32_t kB = smem_u32(smem + kPaK);
 #pragma unroll
-      for (int u = 0; u < 8; ++u)
-        x[u] = (i0 + u < nrows) ? __bfloat162float(*reinterpret_cast<const __nv_bfloat16*>(buf + scr(i0 + u, col)))
-                                : 0.f;
+    for (int kk = 0; kk < D / 16; ++kk) {
+      const uint32_t off = (kk >> 2) * (kPaRows * 128) + (kk & 3) * 32;
+      pa_mma(tS, pa_desc(sQ + off, 16, 1024), pa_desc(kB + off, 16, 1024), pa_idesc(false), kk > 0);
+    }
+    pa_commit(smem_u32(&bars[0]));
+  }
+  const int ti = (row_ok ? r / G : 0) + (tok0 - a0);  // the row's token in the chunk
+  const int sg = s_seg[ti];                            // its segment's first token, or -1
+  const int lo = max(sg, 0);
+  const float rz = s_rz[ti];
+  float cdot = 0.f;  // q . c_k over this half's dims, when the segment runs in from before the chunk
+  if (sg < 0) {
 #pragma unroll
-      for (int u = 0; u < 8; ++u) {
-        const int i = i0 + u;
-        if (i < nrows) {
-          if (s_op[i]) acc = 0.f;
-          acc = fmaf(s_om[i], zero ? 0.f : x[u], acc);
-          // this token's running mean
-          *reinterpret_cast<__nv_bfloat16*>(buf + scr(i, col)) = __float2bfloat16_rn(acc * s_rz[i]);
-        }
-      }
+    for (int jj = 0; jj < 8; ++jj) {
+      const int cj = hf * 8 + jj;
+      float qf[8];
+      Chunk<__nv_bfloat16>::unpack(*reinterpret_cast<const uint4*>(smem + kPaQ + pa_swz(r, cj)), qf);
+#pragma unroll
+      for (int e = 0; e < 8; ++e) cdot = fmaf(qf[e], carry[cj * 8 + e], cdot);
     }
   }
-  __syncthreads();
-
-  // ---- merge the diagonal state and write the row (TMEM loads by every lane)
-  const int ti = (row_ok ? r / G : 0) + (tok0 - a0);  // the token's row in the staged chunk
-  const unsigned char* kt = rk;
-  const unsigned char* vt = rv;
-  float dp = 0.f;
+  wait_bar(0, ntiles & 1);  // S_d is in TMEM
+  tc_fence_after();
+  float wsum = 0.f;
 #pragma unroll
-  for (int j = 0; j < 8; ++j) {
-    const int jj = hf * 8 + j;
-    const uint4 qu = *reinterpret_cast<const uint4*>(smem + kPaQ + pa_swz(r, jj));
-    const uint4 ku = *reinterpret_cast<const uint4*>(kt + scr(ti, jj * 8));
-    float qf[8], kf[8];
-    Chunk<__nv_bfloat16>::unpack(qu, qf);
-    Chunk<__nv_bfloat16>::unpack(ku, kf);
+  for (int c0 = 0; c0 < HALF; c0 += 32) {
+    float f[32];
+    pa_ld32(tS + lane_base + col0 + c0, f);
 #pragma unroll
-    for (int e = 0; e < 8; ++e) dp = fmaf(qf[e], kf[e], dp);
+    for (int i = 0; i < 32; ++i) {
+      const int j = (int)col0 + c0 + i;
+      if (j >= lo && j <= ti) wsum = fmaf(s_om[j], f[i], wsum);
+    }
   }
-  s_x[hf * kPaRows + r] = dp;
-  s_y[hf * kPaRows + r] = l;
+  s_x[hf * kPaRows + r] = wsum + cdot;
   __syncthreads();
-  const float dsc = (dp + s_x[(hf ^ 1) * kPaRows + r]) * qscale;  // k~[0] = 0: q[0] drops out
-  const float lt = l + s_y[(hf ^ 1) * kPaRows + r];
-  const float M = fmaxf(m, dsc);
-  const float cO = (m == -INFINITY) ? 0.f : exp2f(m - M);
-  const float cD = exp2f(dsc - M);
-  const float inv = 1.f / (lt * cO + cD);
+  const float dsc = (s_x[r] + s_x[kPaRows + r]) * rz * qscale;  // the diagonal score (log2 units)
+  {
+    const bool grow = dsc > m + 8.f;
+    const float mn = grow ? dsc : m;
+    const bool resc = grow && m != -INFINITY;
+    const float corr = resc ? pa_ex2(m - mn) : 1.f;
+    l *= corr;
+    if (__any_sync(0xffffffffu, resc)) {
+      for (int c0 = 0; c0 < HALF; c0 += 32) {
+        float f[32];
+        pa_ld32(tO + lane_base + col0 + c0, f);
+#pragma unroll
+        for (int i = 0; i < 32; ++i) f[i] *= corr;
+        pa_st32(tO + lane_base + col0 + c0, f);
+      }
+    }
+    m = mn;
+  }
+  const float pd = pa_ex2(dsc - m);  // the diagonal's weight, below 2^8
+  const float pw = pd * rz;
+  {
+    uint32_t pk[HALF / 2];
+#pragma unroll
+    for (int c0 = 0; c0 < HALF; c0 += 32) {
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        const int j = (int)col0 + c0 + 2 * i;
+        const float p0 = (j >= lo && j <= ti) ? pw * s_om[j] : 0.f;
+        const float p1 = (j + 1 >= lo && j + 1 <= ti) ? pw * s_om[j + 1] : 0.f;
+        pk[c0 / 2 + i] = Chunk<__nv_bfloat16>::pack2(p0, p1);
+      }
+    }
+    float pf[32];
+#pragma unroll
+    for (int i = 0; i < 32; ++i) pf[i] = __uint_as_float(pk[i]);
+    pa_st32(tS + lane_base + col0, pf);
+  }
+  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+  s_y[hf * kPaRows + r] = l + (hf == 0 ? pd : 0.f);  // the row sum, the diagonal counted once
+  tc_fence_before();
+  __syncthreads();
+  if (tid == 0) {
+    tc_fence_after();
+    const uint32_t vB = smem_u32(smem + kPaV);
+#pragma unroll
+    for (int kk = 0; kk < kPaSlots / 16; ++kk) {
+      const uint32_t aT = tS + (uint32_t)((kk >> 2) * HALF + (kk & 3) * 8);
+      pa_mma_ts(tO, aT, pa_desc(vB + kk * 2048, kPaRows * 128, 1024), pa_idesc(true), ntiles > 0 || kk > 0);
+    }
+    pa_commit(smem_u32(&bars[1]));
+  }
+  wait_bar(1, ntiles & 1);
+  tc_fence_after();
+  const float inv = 1.f / (s_y[r] + s_y[kPaRows + r]);
+  const float cw = (sg < 0) ? pw : 0.f;  // weight of the carried value sums
   char* orow = a.out + ((size_t)(row_ok ? tau_r : tok0) * L.Hq + (size_t)h * G + r % G) * ROW;
   for (int c0 = 0; c0 < HALF; c0 += 32) {
     float f[32];
-    if (ntiles > 0) pa_ld32(tO + lane_base + col0 + c0, f);  // CTA-uniform
-    if (ntiles == 0 || m == -INFINITY) {
-#pragma unroll
-      for (int i = 0; i < 32; ++i) f[i] = 0.f;
-    }
+    pa_ld32(tO + lane_base + col0 + c0, f);
     if (row_ok) {
 #pragma unroll
       for (int q4 = 0; q4 < 4; ++q4) {
         const int cc = col0 + c0 + q4 * 8;
-        float vf[8], o[8];
-        Chunk<__nv_bfloat16>::unpack(*reinterpret_cast<const uint4*>(vt + scr(ti, cc)), vf);
+        float o[8];
 #pragma unroll
-        for (int e = 0; e < 8; ++e) o[e] = (f[q4 * 8 + e] * cO + vf[e] * cD) * inv;
+        for (int e = 0; e < 8; ++e) o[e] = fmaf(cw, carry[D + cc + e], f[q4 * 8 + e]) * inv;
         *reinterpret_cast<uint4*>(orow + cc * 2) = Chunk<__nv_bfloat16>::pack(o);
       }
     }
