@@ -18,11 +18,13 @@
 //                      tcgen05.ld of S, the staircase mask (slot < len(i) - 1),
 //                      online softmax in the log2 domain (the halves trade
 //                      their maxima through shared memory), P rounded to bf16
-//                      into shared memory
-//   O += P V           tcgen05.mma with V as an MN-major B operand, into TMEM
-// The diagonal state of each token is rebuilt at the end from the prompt's
-// k, v rows of the token's 128-token chunk and the segment sums the prefill
-// scan recorded at the chunk start ("carry"), then merged into the row.
+//                      and stored over the thread's own S columns in TMEM
+//   O += P V           tcgen05.mma with P read from TMEM and V as an MN-major B
+//                      operand, into TMEM
+// The diagonal state enters as one more tile built from the prompt's k, v rows
+// of the token's 128-token chunk and the segment sums the prefill scan
+// recorded at the chunk start ("carry"): its score is Q Kraw^T summed with the
+// segment's weights, its value P_d Vraw (see the end of the kernel).
 #include <math.h>
 
 #include "dmc_internal.cuh"
