@@ -11,7 +11,11 @@ Modules:
                compressed cache), the closed form of a prompt's slots (segment
                means of Eq. partial-accumulation with binary alpha) and the
                training-time masked formulation (Eq. partial-accumulation plus the
-               additive mask of the masking figure and the masking appendix).
+               additive mask of the masking figure and the masking appendix);
+               prompt-phase attention (each prompt token over the closed slots
+               and its own running state); the window-grouping approximation of
+               Sec. 3.3 (window = w) in the update, the closed form and the
+               masked formulation.
   cref      -- ctypes loader for dmc_ref.c, the same Algorithm 1 plus attention in
                plain C (fp64), used for timed CPU baselines and for parity at sizes
                where numpy's per-token loop is too slow.
