@@ -15,6 +15,16 @@ Recipe per workload (all tensors [tokens, heads, head_dim] row-major):
   q[..., 0] ~ N(0, 1) * scale feeds omega
 Values are drawn in fp32 and then cast, so |k[0]| >= 0.05 holds after the bf16
 cast and no decision sits at the sigmoid tie.
+
+High-signal variant (parity tests only; every workload above leaves it off):
+  q ~ N(0, 1) * q_scale                           a larger query scale makes the
+                                                  softmax peak over a few slots
+  v += N(0, 1) * v_block_offset                   one offset vector per block of
+                                                  16 prompt tokens (per decode
+                                                  token), so slot values and
+                                                  outputs are O(1), not O(1/sqrt n)
+These draws come after the ones above, so a workload with both off draws
+exactly the numbers it always did.
 """
 from __future__ import annotations
 
@@ -58,6 +68,10 @@ class Workload:
     # shared by every head of a layer, so all heads of a sequence have the
     # same segments and lengths
     hardc: bool = False
+    # high-signal parity inputs: query scale (0 = `scale`) and the std of a
+    # per-block offset added to v (0 = none)
+    q_scale: float = 0.0
+    v_block_offset: float = 0.0
 
     @property
     def group(self) -> int:
@@ -137,15 +151,17 @@ def _gen(device, seed):
     return g
 
 
-def _draw_tokens(n, wl: Workload, p_layer, g, device, want_full_q: bool):
-    """Draw n tokens of one layer in fp32: q (full or first neuron), k, v."""
+def _draw_tokens(n, wl: Workload, p_layer, g, device, want_full_q: bool, block: int = 1):
+    """Draw n tokens of one layer in fp32: q (full or first neuron), k, v.
+    `block`: tokens that share one v offset (high-signal variant only)."""
     H, Hq, d, s = wl.num_kv_heads, wl.num_q_heads, wl.head_dim, wl.scale
+    qs = wl.q_scale if wl.q_scale > 0 else s
     k = torch.randn((n, H, d), generator=g, device=device) * s
     v = torch.randn((n, H, d), generator=g, device=device) * s
     if want_full_q:
-        q = torch.randn((n, Hq, d), generator=g, device=device) * s
+        q = torch.randn((n, Hq, d), generator=g, device=device) * qs
     else:
-        q = torch.randn((n, Hq), generator=g, device=device) * s
+        q = torch.randn((n, Hq), generator=g, device=device) * qs
     u = torch.rand((n, H), generator=g, device=device)
     mag = torch.randn((n, H), generator=g, device=device).abs() + 0.1
     p = torch.as_tensor(p_layer, dtype=torch.float32, device=device)
@@ -158,6 +174,10 @@ def _draw_tokens(n, wl: Workload, p_layer, g, device, want_full_q: bool):
             q[:, :] = q[:, :1].clone()
     sign = torch.where(u < p[None, :], -1.0, 1.0)
     k[:, :, 0] = sign * s * mag
+    if wl.v_block_offset > 0 and n > 0:
+        nb = (n + block - 1) // block
+        off = torch.randn((nb, H, d), generator=g, device=device) * wl.v_block_offset
+        v = v + off.repeat_interleave(block, dim=0)[:n]
     return q, k, v
 
 
@@ -187,7 +207,7 @@ def gen_prompt(wl: Workload, layer: int, device, seqs=None, p=None, full_q: bool
     for b, n in zip(seqs, lens):
         n = int(n)
         g = _gen(device, derive_seed(wl.seed, 1, layer, b))
-        qb, kb, vb = _draw_tokens(n, wl, p[layer], g, device, want_full_q=full_q)
+        qb, kb, vb = _draw_tokens(n, wl, p[layer], g, device, want_full_q=full_q, block=16)
         if full_q:
             qf[off:off + n] = qb.to(dt)
             q0[off:off + n] = qb[:, :, 0].to(dt)

@@ -1,0 +1,138 @@
+"""High-signal parity cases for the bf16 attention kernels (GPU).
+
+At the workloads' input scale (q, k, v ~ N(0, 0.25)) the softmax over a
+thousand slots is nearly flat and outputs are O(0.05), so a kernel that
+ignored the query would still land within the bf16 tolerance (2e-2) of the
+oracle. These cases draw inputs whose outputs sit far above it: queries at
+scale 6 over keys at scale 0.5 (a peaked softmax: score std ~3 over up to
+3,200 slots) and values at scale 0.5 plus one offset (std 0.5) per block of 16
+prompt tokens, so slot values and outputs are O(1) but mostly below 2, where a
+bf16 output rounds by at most 0.004. Heads run from a few dozen slots to over
+3,000, split over many workers.
+
+Each case checks, per head:
+  - slot counts, slots, z and every output within 2e-2 of the fp64 oracle
+    (the harness's comparison, Algorithm 1 and Eq. attn-softmax);
+  - every output farther than 2e-2 from each of three mutant oracles (the
+    query ignored, the 1/sqrt(d_h) scale left out, one 32-slot page dropped;
+    tests/mutants.py), so that each mistake would fail the test.
+Covered: the MHA CUDA-core kernel (d 128 and 64, dense and sparse unit
+ranges), the grouped-query mma.sync kernel (G = 2, 4, 8) and the prompt
+attention tcgen05 kernel (G = 1, 2, 4, 8). The observed errors are printed.
+"""
+import numpy as np
+import pytest
+import torch
+
+from oracle import cref
+from paper_2403_09636_gb300 import synthetic as S
+from tests import dmc_harness as H
+from tests import mutants as M
+
+pytestmark = pytest.mark.gpu
+TOL = 2e-2
+
+
+def _wl(name, layers, B, Hq, Hkv, d, prompt, steps, cr, seed):
+    return S.Workload(name, layers, B, Hq, Hkv, d, "bf16", prompt, steps, cr, 0.5, seed=seed,
+                      q_scale=6.0, v_block_offset=0.5)
+
+
+DECODE = [
+    # 64 long MHA heads (1,200-3,200 slots): more units than warps, every head
+    # split over ~35 workers
+    _wl("sig_mha_dense", 1, 8, 8, 8, 128, (1200, 3200), 12, ("choice", (1.0, 1.5)), 300),
+    # short and long heads over two layers, fewer units than warps
+    _wl("sig_mha_mixed", 2, 4, 4, 4, 128, (20, 2600), 16, ("choice", (1.0, 2.0, 4.0)), 301),
+    _wl("sig_mha_d64", 1, 3, 6, 6, 64, (30, 2400), 16, ("choice", (1.0, 2.0)), 302),
+    _wl("sig_gqa_g2", 1, 4, 8, 4, 128, (20, 2600), 16, ("choice", (1.0, 2.0)), 303),
+    _wl("sig_gqa_g4", 1, 4, 16, 4, 128, (20, 2600), 16, ("choice", (1.0, 2.0)), 304),
+    _wl("sig_gqa_g8", 1, 4, 32, 4, 128, (20, 2600), 16, ("choice", (1.0, 2.0)), 305),
+    _wl("sig_gqa_g4_d64", 1, 4, 8, 2, 64, (20, 2600), 16, ("choice", (1.0, 2.0)), 306),
+    # 32 long grouped heads: more units than the tensor-core kernel's warps
+    _wl("sig_gqa_g8_dense", 1, 8, 32, 4, 128, (1500, 3000), 12, ("fixed", 1.0), 307),
+]
+
+
+def _separation_failures(tag, got, muts, n_slots):
+    """Per head: every mutant farther than TOL, except that a head of one
+    page (<= 32 slots) has no page to drop."""
+    sep = M.separation(got, muts)
+    modes = [m for m in M.MODES if m != "droppage" or n_slots > M.PAGE]
+    return sep, [f"{tag}: within {sep[m]:.4f} of the '{m}' mutant" for m in modes
+                 if not sep[m] > TOL]
+
+
+@pytest.mark.parametrize("wl", DECODE, ids=lambda w: w.name)
+def test_decode_high_signal_separates_mutants(cuda_dev, wl):
+    run = H.Run(wl, cuda_dev, H.all_samples(wl))
+    assert run.len_ok, run.len_msgs[:5]
+    bad = run.compare(tol=TOL)
+    ref = run.oracle()
+    worst = {"oracle": 0.0, "out_max": 0.0, **{m: np.inf for m in M.MODES}}
+    for s in run.samples:
+        I = run.inst[s]
+        got = np.array(I["out"])                                   # [S, G, d]
+        muts = M.decode_outputs(I["k_prompt"], I["v_prompt"], I["q0_prompt"],
+                                np.array(I["k_dec"]), np.array(I["v_dec"]), np.array(I["q_dec"]))
+        worst["oracle"] = max(worst["oracle"], float(np.max(np.abs(got - ref[s]["out"]))))
+        worst["out_max"] = max(worst["out_max"], float(np.max(np.abs(ref[s]["out"]))))
+        sep, fails = _separation_failures(str(s), got, muts, int(ref[s]["len"]))
+        for m in M.MODES:
+            if m != "droppage" or int(ref[s]["len"]) > M.PAGE:
+                worst[m] = min(worst[m], sep[m])
+        bad += fails
+    print(f"\n{wl.name}: max |gpu - oracle| {worst['oracle']:.5f}, max |out| {worst['out_max']:.3f}, "
+          "min |gpu - mutant| " + ", ".join(f"{m} {worst[m]:.4f}" for m in M.MODES))
+    assert not bad, bad[:10]
+
+
+PROMPT = [
+    _wl(f"sig_prompt_g{G}", 1, 3, 2 * G, 2, 128, (30, 2200), 0, ("choice", (1.0, 2.0, 4.0)), 310 + G)
+    for G in (1, 2, 4, 8)
+]
+
+
+@pytest.mark.parametrize("wl", PROMPT, ids=lambda w: w.name)
+def test_prompt_attention_high_signal_separates_mutants(cuda_dev, wl):
+    G = wl.group
+    lens = S.prompt_lengths(wl)
+    cache = H.cache_for(wl, cuda_dev)
+    pr = S.gen_prompt(wl, 0, cuda_dev, full_q=True)
+    out = torch.full_like(pr["q"], float("nan"))
+    cache.prefill_attention(0, pr["q"], pr["k"], pr["v"], pr["cu_seqlens"], pr["max_seqlen"], out)
+    assert cache.status()[:2] == (0, 0)
+    cu = pr["cu_seqlens"].cpu().numpy()
+    f = lambda t: t.float().cpu().numpy()
+    heads, where = [], []
+    for b in range(wl.batch):
+        sl = slice(int(cu[b]), int(cu[b + 1]))
+        for h in range(wl.num_kv_heads):
+            heads.append({"k_prompt": np.zeros((0, 128)), "v_prompt": np.zeros((0, 128)),
+                          "q0_prompt": np.zeros((0, G)), "k_dec": f(pr["k"][sl, h]),
+                          "v_dec": f(pr["v"][sl, h]), "q_dec": f(pr["q"][sl, h * G:(h + 1) * G])})
+            where.append((b, h, sl))
+    ref = cref.run_heads(heads, threads=8)
+    got_len = cache.lengths(0).cpu().numpy()
+    bad = []
+    worst = {"oracle": 0.0, "out_max": 0.0, **{m: np.inf for m in M.MODES}}
+    for (b, h, sl), hd, r in zip(where, heads, ref):
+        if got_len[b, h] != r["len"]:
+            bad.append(f"len b{b} h{h}: {got_len[b, h]} != {r['len']}")
+            continue
+        got = f(out[sl, h * G:(h + 1) * G])
+        err = float(np.max(np.abs(got - r["out"])))
+        worst["oracle"] = max(worst["oracle"], err)
+        worst["out_max"] = max(worst["out_max"], float(np.max(np.abs(r["out"]))))
+        if not err <= TOL:
+            bad.append(f"out b{b} h{h}: {err}")
+        muts = M.prompt_outputs(hd["k_dec"], hd["v_dec"], hd["q_dec"])
+        sep, fails = _separation_failures(f"b{b} h{h} ({int(lens[b])} tokens)", got, muts,
+                                          int(r["len"]))
+        for m in M.MODES:
+            if m != "droppage" or int(r["len"]) > M.PAGE:
+                worst[m] = min(worst[m], sep[m])
+        bad += fails
+    print(f"\n{wl.name}: max |gpu - oracle| {worst['oracle']:.5f}, max |out| {worst['out_max']:.3f}, "
+          "min |gpu - mutant| " + ", ".join(f"{m} {worst[m]:.4f}" for m in M.MODES))
+    assert not bad, bad[:10]
