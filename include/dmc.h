@@ -167,18 +167,28 @@ dmc_status dmc_decode_step(dmc_cache_t cache, int32_t layer, const void* q_dev,
  * device memory of their own: a plugin or custom operator that a host
  * framework hands only its input and output buffers (the framework owns every
  * allocation), or a latency-critical loop that must not pay cudaMalloc's
- * implicit device synchronisation. Same arguments, semantics and results as
+ * implicit device synchronisation. Same arguments and semantics as
  * dmc_decode_step; it allocates nothing and calls no allocating routine.
  * The scratch is the split-K partial softmax states of one launch, kept in a
- * file-scope __device__ array of 4.33 MB (2 states of head_dim + 4 floats for
- * each of at most 4096 worker warps) that every GPU loading the library holds
- * until the process exits; a cache whose decode grid would need more returns
- * DMC_ERR_INVALID_ARG. Nothing in it needs to start at zero: each launch writes
- * every state before reading it. The first call on a device looks up the
- * array's device address on that device (which must be current and be the
- * cache's device); make that first call before any stream capture. All calls
- * share the one array, so calls whose launches overlap on the GPU (any caches,
- * any streams) race and must be ordered by the caller. */
+ * file-scope __device__ array of 8 MiB (2,097,152 floats) that every GPU
+ * loading the library holds until the process exits. One launch needs
+ *   2 * grid * 8 states of head_dim + 4 floats   (CUDA-core kernel: MHA, fp32,
+ *                                                 groups above 8), or
+ *   2 * grid * 6 * G states of head_dim + 2 floats (tensor-core kernel: bf16
+ *                                                 groups of 2 to 8 queries),
+ * grid being the cache's decode grid (at most one or two blocks per SM). Every
+ * MHA grid fits; a tensor-core grid of group 8 and head_dim 128 fits up to 168
+ * blocks (a GB300 runs 152). A grid that does not fit is cut to the blocks
+ * that do: the work split follows the grid, so the results then differ from
+ * dmc_decode_step's only by the rounding of the split-K sums; when it fits,
+ * they are bit-identical. Nothing in the array needs to start at zero: each
+ * launch writes every state before reading it. The first call on a device
+ * looks up the array's device address on that device (which must be current
+ * and be the cache's device) and keeps it for the life of the process, so the
+ * device must not be reset (cudaDeviceReset) after that call, and the first
+ * call should come before any stream capture. All calls share the one array,
+ * so calls whose launches overlap on the GPU (any caches, any streams) race
+ * and must be ordered by the caller. */
 dmc_status dmc_decode_step_static_scratch(dmc_cache_t cache, int32_t layer, const void* q_dev,
                                           const void* k_dev, const void* v_dev, void* out_dev,
                                           cudaStream_t stream);

@@ -329,17 +329,27 @@ dmc_status dmc_decode_step_static_scratch(dmc_cache_t c, int32_t layer, const vo
   size_t floats = 0;
   e = dmc::decode_static_partials(dev, &scratch, &floats);
   if (e != cudaSuccess) return DMC_ERR_CUDA;
-  // the launch's partial states (head_dim + 4 floats each for the CUDA-core
-  // kernel, head_dim + 2 for the tensor-core kernel) must fit
-  const size_t fit = floats / (size_t)(L.D + (c->gqa ? 2 : 4));
-  if ((size_t)c->plan.partial_states > fit) return DMC_ERR_INVALID_ARG;
+  // One launch writes two partial states per worker warp: of head_dim + 4
+  // floats for the CUDA-core kernel (8 warps per block), and one per query
+  // of the group, of head_dim + 2 floats, for the tensor-core kernel (6 warps
+  // per block). A grid that needs more than the array holds is cut to fit;
+  // the work split follows the grid, so results differ from dmc_decode_step's
+  // only by the order of the split-K sums.
+  const size_t state_floats = (size_t)L.D + (c->gqa ? 2 : 4);
+  const size_t per_block = (size_t)2 * (c->gqa ? dmc::kGqaWarpsPerBlock : dmc::kDecodeWarpsPerBlock) *
+                           (c->gqa ? L.G : 1);
+  const size_t fit_blocks = floats / state_floats / per_block;
+  if (fit_blocks < 1) return DMC_ERR_INVALID_ARG;
+  dmc::DecodePlan plan = c->plan;
+  if ((size_t)plan.grid > fit_blocks) plan.grid = (int)fit_blocks;
+  plan.partial_states = (int)(per_block * plan.grid);
   Layout ls = L;
   ls.partials = scratch;
-  ls.partial_cap = (int)fit;
+  ls.partial_cap = (int)(floats / state_floats);
   const bool pdl = use_pdl(c, layer);
   if (c->gqa)
-    return cuda_status(dmc::gqa_launch(ls, layer, c->plan, pdl, q_dev, k_dev, v_dev, out_dev, stream));
-  return cuda_status(dmc::decode_launch(ls, layer, c->Gv, c->plan, pdl, q_dev, k_dev, v_dev,
+    return cuda_status(dmc::gqa_launch(ls, layer, plan, pdl, q_dev, k_dev, v_dev, out_dev, stream));
+  return cuda_status(dmc::decode_launch(ls, layer, c->Gv, plan, pdl, q_dev, k_dev, v_dev,
                                         out_dev, stream));
 }
 

@@ -43,7 +43,7 @@
 
 namespace dmc {
 
-constexpr int kWarps = 8;  // independent workers per block
+constexpr int kWarps = kDecodeWarpsPerBlock;  // independent workers per block
 constexpr int kDecodeThreads = kWarps * 32;
 constexpr int kRing = 6;        // quads per warp ring (kRing - 1 in flight)
 constexpr int kWindow = 64;     // page units per warp window (page id + rows to copy)
@@ -791,11 +791,15 @@ cudaError_t decode_launch(const Layout& L, int layer, int Gv, const DecodePlan& 
 }
 
 // ---------------------------------------------------------------- static scratch
-// Scratch of dmc_decode_step_static_scratch: room for the split-K partial
-// softmax states of one launch (2 per worker warp, head_dim <= 128, at most
-// 512 blocks of 8 warps), 4.33 MB. Every GPU that loads the library holds it
-// until exit.
-constexpr size_t kStaticPartialFloats = (size_t)2 * kMaxWorkers * kPartialStride<128>;
+// Scratch of dmc_decode_step_static_scratch: the split-K partial softmax states
+// of one launch, 8 MiB. That holds two states of head_dim + 4 floats for each
+// of the MHA kernel's 4096 worker warps at most, and the tensor-core kernel's
+// two states per query of a group of 8 (head_dim + 2 floats each) for up to
+// 168 blocks of 6 warps (a GB300 runs 152). Every GPU that loads the library
+// holds it until exit.
+constexpr size_t kStaticPartialFloats = (size_t)2 << 20;
+static_assert(kStaticPartialFloats >= (size_t)2 * kMaxWorkers * kPartialStride<128>,
+              "the static scratch holds every MHA decode grid");
 static __device__ __align__(256) float g_decode_static_partials[kStaticPartialFloats];
 
 // Host code must not pass g_decode_static_partials itself to a kernel (on the

@@ -32,7 +32,7 @@
 
 namespace dmc {
 
-constexpr int kGWarps = 6;  // workers per block
+constexpr int kGWarps = kGqaWarpsPerBlock;  // workers per block
 constexpr int kGThreads = kGWarps * 32;
 constexpr int kGRing = 4;     // tiles per warp ring (kGRing - 1 in flight)
 constexpr int kTile = 16;     // slots per tile
