@@ -13,6 +13,8 @@ constexpr int kPage = 32;              // slots per page (the paper's page size)
 constexpr int kPrefillChunk = 128;     // prompt tokens per prefill block
 constexpr int kMaxVirtualHeads = 16384;
 constexpr int kMaxWindow = 32;         // longest window of the window-grouping approximation
+constexpr int kDecodeWarpsPerBlock = 8;  // worker warps per block, CUDA-core decode kernel
+constexpr int kGqaWarpsPerBlock = 6;     // worker warps per block, tensor-core decode kernel
 
 // Device-side view of one cache. Passed by value to every kernel.
 struct Layout {
@@ -103,7 +105,7 @@ template <> struct Chunk<__nv_bfloat16> {
 
 __device__ __forceinline__ float sigmoidf_(float x) { return 1.0f / (1.0f + __expf(-x)); }
 
-// ---------------------------------------------------------------- PTX: mbarrier + bulk copy
+// ---------------------------------------------------------------- PTX: mbarrier, cp.async, mma
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
@@ -149,7 +151,12 @@ __device__ __forceinline__ uint64_t globaltimer_ns() {
   return t;
 }
 
-constexpr uint64_t kWaitLimitNs = 2000000000ull;  // 2 s: normal waits take microseconds
+// Longest in-kernel wait before it gives up. Normal waits take microseconds;
+// a build of a test kernel may shorten the limit.
+#ifndef DMC_WAIT_LIMIT_NS
+#define DMC_WAIT_LIMIT_NS 2000000000ull  // 2 s
+#endif
+constexpr uint64_t kWaitLimitNs = DMC_WAIT_LIMIT_NS;
 
 // Waits for the phase with the given parity to complete. Gives up after
 // kWaitLimitNs, sets DMC_FAULT_WAIT_TIMEOUT and returns false.
@@ -166,17 +173,6 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, unsigne
       return false;
     }
   }
-}
-
-// One TMA bulk copy global -> this CTA's shared memory, completing on `bar`.
-// dst, src 16-byte aligned; bytes a multiple of 16.
-__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t bytes,
-                                         uint32_t bar) {
-  asm volatile(
-      "cp.async.bulk.shared::cta.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-          dst),
-      "l"(src), "r"(bytes), "r"(bar)
-      : "memory");
 }
 
 // cp.async (LDGSTS) of 16 bytes, L2 only, into this thread's shared memory.

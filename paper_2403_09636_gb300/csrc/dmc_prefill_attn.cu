@@ -162,6 +162,7 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
 
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kPaMisc);  // [0] S done, [1] O done
   uint32_t* tslot = reinterpret_cast<uint32_t*>(smem + kPaMisc + 16);
+  volatile int* s_abort = reinterpret_cast<volatile int*>(smem + kPaMisc + 32);  // a wait gave up
   int* s_len = reinterpret_cast<int*>(smem + kPaMisc + 64);            // [128] slots after token
   float* s_om = reinterpret_cast<float*>(smem + kPaMisc + 64 + 512);   // [128] omega
   float* s_rz = reinterpret_cast<float*>(smem + kPaMisc + 64 + 1024);  // [128] 1 / z after token
@@ -268,9 +269,10 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
     }
   }
   if (tid == 0) {
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(&bars[0])));
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(&bars[1])));
-    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    mbar_init(smem_u32(&bars[0]), 1);
+    mbar_init(smem_u32(&bars[1]), 1);
+    fence_mbar_init();
+    *s_abort = 0;
   }
   if (warp == 0) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
@@ -317,18 +319,21 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
   const uint32_t col0 = hf * HALF;                                // this thread's first column
   const float qscale = 1.4426950408889634f / sqrtf((float)D);   // log2(e) / sqrt(d_h)
 
+  // Waits for a tensor-core commit. A wait that gives up (mbar_wait sets the
+  // fault bit) raises s_abort; later waits then return at once, and the block
+  // leaves at the next point where every thread has passed a barrier after
+  // the wait: no further MMA is issued, its copies drain, TMEM is freed.
   auto wait_bar = [&](int which, int ph) {
-    const uint32_t bar = smem_u32(&bars[which]);
-#pragma unroll 1
-    for (int i = 0; i < 64; ++i)
-      if (mbar_try_wait(bar, ph)) return;
-    const uint64_t tb = globaltimer_ns();
-#pragma unroll 1
-    while (!mbar_try_wait(bar, ph)) {
-      if (globaltimer_ns() - tb > kWaitLimitNs) {
-        atomicOr(L.error, DMC_FAULT_WAIT_TIMEOUT);
-        return;
-      }
+    if (*s_abort) return;
+    if (!mbar_wait(smem_u32(&bars[which]), ph, L.error)) *s_abort = 1;
+  };
+  auto leave = [&]() {
+    cp_async_wait<0>();
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) {
+      tc_fence_after();
+      asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(256));
     }
   };
 
@@ -343,6 +348,7 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
     cp_async_wait<1>();  // Q and K(jt) have landed (this thread's copies)
     fence_async_smem();
     __syncthreads();
+    if (*s_abort) break;  // uniform: every wait that could raise it is behind the barrier
     if (tid == 0) {
       tc_fence_after();
       const uint32_t kA = sQ, kB = smem_u32(smem + kPaK);
@@ -379,6 +385,7 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
     }
     s_x[hf * kPaRows + r] = mx * qscale;  // qscale > 0
     __syncthreads();
+    if (*s_abort) break;
     const float mt = fmaxf(mx * qscale, s_x[(hf ^ 1) * kPaRows + r]);  // the tile's row maximum
     const bool grow = mt > m + 8.f;  // false while the row has seen nothing
     const float mn = grow ? mt : m;
@@ -454,6 +461,10 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
   cp_async_wait<0>();
   tc_fence_after();
   __syncthreads();  // every MMA and copy of the loop is over: the K and V buffers are free
+  if (*s_abort) {
+    leave();
+    return;
+  }
 
   // ---- the diagonal state as one more tile. When token i of the chunk
   // attends, its own slot holds k~ = (c_k [no opening in the chunk up to i] +
@@ -520,6 +531,10 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
   }
   s_x[hf * kPaRows + r] = wsum + cdot;
   __syncthreads();
+  if (*s_abort) {
+    leave();
+    return;
+  }
   const float dsc = (s_x[r] + s_x[kPaRows + r]) * rz * qscale;  // the diagonal score (log2 units)
   {
     const bool grow = dsc > m + 8.f;
