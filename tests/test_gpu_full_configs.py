@@ -26,17 +26,17 @@ CASES = ["llama2_7b_4x", "llama2_7b_mixed", "llama2_13b_4x", "llama2_70b_gqa_2x"
 def test_full_size_sampled(cuda_dev, name):
     wl = S.WORKLOADS[name]
     wl, cache = H.full_size_cache(wl, cuda_dev, wl.decode_steps)
-    if wl.num_layers < S.WORKLOADS[name].num_layers:
-        print(f"{name}: {wl.num_layers} of {S.WORKLOADS[name].num_layers} layers fit the device")
+    covered = f"{name}: {wl.num_layers} of {S.WORKLOADS[name].num_layers} layers checked"
+    print(f"\n{covered}")
     run = H.Run(wl, cuda_dev, H.random_samples(wl, 64, seed=17), cache=cache)
-    assert run.len_ok, run.len_msgs[:5]
+    assert run.len_ok, (covered, run.len_msgs[:5])
     if wl.hardc:
         # DMC-HardC: every head of a sequence holds the same number of slots
         for layer in range(wl.num_layers):
             ln = cache.lengths(layer)
-            assert bool((ln == ln[:, :1]).all()), layer
+            assert bool((ln == ln[:, :1]).all()), (covered, layer)
     bad = run.compare()
-    assert not bad, bad[:10]
+    assert not bad, (covered, bad[:10])
     del run, cache
     import torch
     torch.cuda.empty_cache()
