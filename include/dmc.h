@@ -162,6 +162,21 @@ dmc_status dmc_decode_step(dmc_cache_t cache, int32_t layer, const void* q_dev,
                            const void* k_dev, const void* v_dev, void* out_dev,
                            cudaStream_t stream);
 
+/* dmc_decode_step for the layers [first_layer, first_layer + num_layers) in
+ * one launch, when the inputs of all of them are ready (the step of each layer
+ * reads only that layer's cache and inputs, Algorithm 1 and Eq. attn-softmax
+ * per KV head, so the layers are independent). Same result for every layer as
+ * calling dmc_decode_step on the layers in order; what it saves is one launch
+ * and one kernel start-up and tail per layer, which dominate small caches.
+ *   q_dev:   [num_layers, batch, num_q_heads, head_dim]
+ *   k_dev, v_dev: [num_layers, batch, num_kv_heads, head_dim]
+ *   out_dev: [num_layers, batch, num_q_heads, head_dim] (written)
+ * Grouped bf16 queries of 2 to 8 per KV head (the tensor-core kernel) are
+ * issued as one launch per layer. num_layers = 0 is a no-op. */
+dmc_status dmc_decode_step_layers(dmc_cache_t cache, int32_t first_layer, int32_t num_layers,
+                                  const void* q_dev, const void* k_dev, const void* v_dev,
+                                  void* out_dev, cudaStream_t stream);
+
 /* dmc_decode_step with its scratch in the library's own static device memory.
  * The paper has no counterpart; this exists for callers that cannot allocate
  * device memory of their own: a plugin or custom operator that a host

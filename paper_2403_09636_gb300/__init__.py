@@ -31,7 +31,7 @@ PAGE_SIZE = 32
 
 EXPORTED = ("dmc_cache_required_bytes", "dmc_cache_create", "dmc_cache_destroy",
             "dmc_cache_reset", "dmc_prefill_compress", "dmc_prefill_attention", "dmc_decode_step",
-            "dmc_decode_step_static_scratch", "dmc_cache_lengths",
+            "dmc_decode_step_layers", "dmc_decode_step_static_scratch", "dmc_cache_lengths",
             "dmc_cache_export_heads", "dmc_cache_status", "dmc_status_string")
 
 
@@ -72,6 +72,7 @@ def lib():
                                                i32, vp]),
             "dmc_prefill_attention": (C.c_int, [vp, i32, i32, i32, vp, vp, vp, vp, i32, i32, vp, vp]),
             "dmc_decode_step": (C.c_int, [vp, i32, vp, vp, vp, vp, vp]),
+            "dmc_decode_step_layers": (C.c_int, [vp, i32, i32, vp, vp, vp, vp, vp]),
             "dmc_decode_step_static_scratch": (C.c_int, [vp, i32, vp, vp, vp, vp, vp]),
             "dmc_cache_lengths": (C.c_int, [vp, i32, vp, vp]),
             "dmc_cache_export_heads": (C.c_int, [vp, i32, i32, vp, i32, vp, vp, vp, vp, vp]),
@@ -122,6 +123,12 @@ def dmc_prefill_attention(handle, layer, first_seq, num_seqs, q_ptr, k_ptr, v_pt
 
 def dmc_decode_step(handle, layer, q_ptr, k_ptr, v_ptr, out_ptr, stream) -> int:
     return lib().dmc_decode_step(handle, layer, q_ptr, k_ptr, v_ptr, out_ptr, stream)
+
+
+def dmc_decode_step_layers(handle, first_layer, num_layers, q_ptr, k_ptr, v_ptr, out_ptr,
+                           stream) -> int:
+    return lib().dmc_decode_step_layers(handle, first_layer, num_layers, q_ptr, k_ptr, v_ptr,
+                                        out_ptr, stream)
 
 
 def dmc_decode_step_static_scratch(handle, layer, q_ptr, k_ptr, v_ptr, out_ptr, stream) -> int:
@@ -223,6 +230,12 @@ class DmcCache:
     def decode(self, layer, q, k, v, out, stream=None):
         _check(dmc_decode_step(self.handle, layer, q.data_ptr(), k.data_ptr(), v.data_ptr(),
                                out.data_ptr(), self._s(stream)), "dmc_decode_step")
+
+    def decode_layers(self, first_layer, q, k, v, out, stream=None):
+        """q, out: [n, B, Hq, D]; k, v: [n, B, Hkv, D] for layers first_layer .. + n - 1."""
+        _check(dmc_decode_step_layers(self.handle, first_layer, q.shape[0], q.data_ptr(),
+                                      k.data_ptr(), v.data_ptr(), out.data_ptr(), self._s(stream)),
+               "dmc_decode_step_layers")
 
     def lengths(self, layer, stream=None):
         t = self.torch

@@ -10,8 +10,8 @@
 
 namespace dmc {
 cudaError_t decode_setup(const Layout& L, int Gv, DecodePlan* plan);
-cudaError_t decode_launch(const Layout& L, int layer, int Gv, const DecodePlan& plan, bool pdl,
-                          const void* q, const void* k, const void* v, void* out,
+cudaError_t decode_launch(const Layout& L, int layer0, int nlayers, int Gv, const DecodePlan& plan,
+                          bool pdl, const void* q, const void* k, const void* v, void* out,
                           cudaStream_t stream);
 cudaError_t prefill_launch(const Layout& L, int layer, int first_seq, int num_seqs, const void* q,
                            long long q_tok, long long q_head, const void* k, const void* v,
@@ -43,7 +43,7 @@ struct dmc_cache {
   int Gv;
   bool gqa;  // grouped queries on the tensor-core kernel (one worker per KV head)
   dmc::DecodePlan plan;
-  int last_decode_layer;  // layer of the latest kernel if it was a decode, else -1
+  int last_decode_lo, last_decode_hi;  // layers [lo, hi) of the latest kernel if it was a decode, else empty
   char* meta;  // lengths, ctl, counters, pool top, error: cleared by create / reset
   size_t meta_bytes;
   float* carry;  // segment sums at prompt chunk starts (prompt attention)
@@ -99,10 +99,18 @@ Offsets offsets(const dmc_cache_config* c) {
   o.pool_top = at; at = align_up(at + 8);
   o.error = at; at = align_up(at + 4);
   o.meta_end = at;
-  o.partials = at; at = align_up(at + dmc::partial_states_cap(G) * (c->head_dim + 4) * 4);
-  o.pending = at; at = align_up(at + (G > 1 ? (size_t)NH * 2 * row : 0));
-  o.pending_at = at; at = align_up(at + (G > 1 ? (size_t)NH * 4 : 0));
-  o.pending_z = at; at = align_up(at + (G > 1 ? (size_t)NH * 4 : 0));
+  // The CUDA-core decode kernel (every cache but grouped bf16 queries of 2 to
+  // 8 per KV head, which run on the tensor-core kernel) keeps its split-K
+  // states and pending rows per layer: one launch may walk several layers
+  // whose blocks run at their own pace.
+  const bool cuda_core = !(c->dtype == DMC_BF16 && G >= 2 && G <= 8);
+  const size_t state_layers = cuda_core ? (size_t)c->num_layers : 1;
+  o.partials = at;
+  at = align_up(at + state_layers * dmc::partial_states_cap(cuda_core ? 1 : G) * (c->head_dim + 4) * 4);
+  const size_t pend = (cuda_core && G > 1) ? (size_t)c->num_layers * NH : 0;
+  o.pending = at; at = align_up(at + pend * 2 * row);
+  o.pending_at = at; at = align_up(at + pend * 4);
+  o.pending_z = at; at = align_up(at + pend * 4);
   o.opens = at; at = align_up(at + (size_t)c->max_prefill_tokens * c->num_kv_heads);
   o.plan = at; at = align_up(at + (size_t)c->num_kv_heads * o.plan_stride * 4);
   o.carry = at; at = align_up(at + (size_t)o.plan_stride * c->num_kv_heads * (2 * c->head_dim + 1) * 4);
@@ -198,7 +206,9 @@ dmc_status dmc_cache_create(const dmc_cache_config* cfg, void* arena_dev, size_t
   L.pool_top = reinterpret_cast<unsigned long long*>(base + o.pool_top);
   L.error = reinterpret_cast<unsigned int*>(base + o.error);
   L.partials = reinterpret_cast<float*>(base + o.partials);
-  L.partial_cap = (int)dmc::partial_states_cap(L.G);
+  const bool cuda_core = !(cfg->dtype == DMC_BF16 && L.G >= 2 && L.G <= 8);
+  L.partial_cap = (int)dmc::partial_states_cap(cuda_core ? 1 : L.G);
+  L.partials_layer_stride = cuda_core ? (long long)L.partial_cap * (L.D + 4) : 0;
   L.opens = reinterpret_cast<unsigned char*>(base + o.opens);
   L.plan = reinterpret_cast<int*>(base + o.plan);
   L.plan_stride = o.plan_stride;
@@ -215,7 +225,7 @@ dmc_status dmc_cache_create(const dmc_cache_config* cfg, void* arena_dev, size_t
   // entry of the CUDA-core kernel (G = 1 for MHA).
   c->gqa = dmc::gqa_supported(L);
   c->Gv = c->gqa ? 1 : L.G;
-  c->last_decode_layer = -1;
+  c->last_decode_lo = c->last_decode_hi = 0;
   cudaError_t e = cudaGetDevice(&c->device);
   if (e == cudaSuccess) e = c->gqa ? dmc::gqa_setup(L, &c->plan) : dmc::decode_setup(L, c->Gv, &c->plan);
   if (e == cudaSuccess) e = cudaMemsetAsync(c->meta, 0, c->meta_bytes, stream);
@@ -229,13 +239,16 @@ dmc_status dmc_cache_create(const dmc_cache_config* cfg, void* arena_dev, size_t
 
 // A decode launch may overlap the tail of the kernel before it on the stream
 // (programmatic dependent launch) only if that kernel was this cache's decode
-// of another layer: its prologue reads the layer's slot counts, page table and
-// pages, which this cache's prefill and decode of the same layer write.
-bool use_pdl(dmc_cache* c, int layer) {
-  const bool pdl = c->last_decode_layer >= 0 && c->last_decode_layer != layer;
-  c->last_decode_layer = layer;
+// of other layers: its prologue reads the first layer's slot counts, page table
+// and pages, which this cache's prefill and decode of that layer write.
+bool use_pdl(dmc_cache* c, int layer0, int nlayers) {
+  const bool pdl = c->last_decode_hi > c->last_decode_lo &&
+                   (layer0 < c->last_decode_lo || layer0 >= c->last_decode_hi);
+  c->last_decode_lo = layer0;
+  c->last_decode_hi = layer0 + nlayers;
   return pdl;
 }
+void no_pdl_next(dmc_cache* c) { c->last_decode_lo = c->last_decode_hi = 0; }
 
 dmc_status dmc_cache_destroy(dmc_cache_t cache) {
   delete cache;
@@ -244,7 +257,7 @@ dmc_status dmc_cache_destroy(dmc_cache_t cache) {
 
 dmc_status dmc_cache_reset(dmc_cache_t c, cudaStream_t stream) {
   if (!c) return DMC_ERR_INVALID_ARG;
-  c->last_decode_layer = -1;
+  no_pdl_next(c);
   return cuda_status(cudaMemsetAsync(c->meta, 0, c->meta_bytes, stream));
 }
 
@@ -263,7 +276,7 @@ dmc_status dmc_prefill_compress(dmc_cache_t c, int32_t layer, int32_t first_seq,
   if (!q_dev || !k_dev || !v_dev || !cu_seqlens_dev || !aligned16(k_dev) || !aligned16(v_dev))
     return DMC_ERR_INVALID_ARG;
   if (q_token_stride < 0 || q_head_stride < 0) return DMC_ERR_INVALID_ARG;
-  c->last_decode_layer = -1;
+  no_pdl_next(c);
   return cuda_status(dmc::prefill_launch(L, layer, first_seq, num_seqs, q_dev, q_token_stride,
                                          q_head_stride, k_dev, v_dev, cu_seqlens_dev, total_tokens,
                                          max_seqlen, nullptr, stream));
@@ -286,7 +299,7 @@ dmc_status dmc_prefill_attention(dmc_cache_t c, int32_t layer, int32_t first_seq
   if (!q_dev || !k_dev || !v_dev || !cu_seqlens_dev || !out_dev || !aligned16(q_dev) ||
       !aligned16(k_dev) || !aligned16(v_dev) || !aligned16(out_dev))
     return DMC_ERR_INVALID_ARG;
-  c->last_decode_layer = -1;
+  no_pdl_next(c);
   const long long q_tok = (long long)L.Hq * L.D, q_head = L.D;
   cudaError_t e = dmc::prefill_launch(L, layer, first_seq, num_seqs, q_dev, q_tok, q_head, k_dev,
                                       v_dev, cu_seqlens_dev, total_tokens, max_seqlen, c->carry,
@@ -305,11 +318,40 @@ dmc_status dmc_decode_step(dmc_cache_t c, int32_t layer, const void* q_dev, cons
   if (!aligned16(q_dev) || !aligned16(k_dev) || !aligned16(v_dev) || !aligned16(out_dev) ||
       !q_dev || !k_dev || !v_dev || !out_dev)
     return DMC_ERR_INVALID_ARG;
-  const bool pdl = use_pdl(c, layer);
+  const bool pdl = use_pdl(c, layer, 1);
   if (c->gqa)
     return cuda_status(dmc::gqa_launch(L, layer, c->plan, pdl, q_dev, k_dev, v_dev, out_dev, stream));
-  return cuda_status(dmc::decode_launch(L, layer, c->Gv, c->plan, pdl, q_dev, k_dev, v_dev,
+  return cuda_status(dmc::decode_launch(L, layer, 1, c->Gv, c->plan, pdl, q_dev, k_dev, v_dev,
                                         out_dev, stream));
+}
+
+dmc_status dmc_decode_step_layers(dmc_cache_t c, int32_t first_layer, int32_t num_layers,
+                                  const void* q_dev, const void* k_dev, const void* v_dev,
+                                  void* out_dev, cudaStream_t stream) {
+  if (!c) return DMC_ERR_INVALID_ARG;
+  const Layout& L = c->lay;
+  if (first_layer < 0 || num_layers < 0 || first_layer + num_layers > L.L) return DMC_ERR_INVALID_ARG;
+  if (num_layers == 0) return DMC_OK;
+  if (!aligned16(q_dev) || !aligned16(k_dev) || !aligned16(v_dev) || !aligned16(out_dev) ||
+      !q_dev || !k_dev || !v_dev || !out_dev)
+    return DMC_ERR_INVALID_ARG;
+  if (c->gqa) {
+    // grouped queries on the tensor cores: one launch per layer
+    const size_t q_ls = (size_t)L.B * L.Hq * L.row_bytes, kv_ls = (size_t)L.B * L.Hkv * L.row_bytes;
+    for (int i = 0; i < num_layers; ++i) {
+      const int layer = first_layer + i;
+      const bool pdl = use_pdl(c, layer, 1);
+      const cudaError_t e = dmc::gqa_launch(
+          L, layer, c->plan, pdl, static_cast<const char*>(q_dev) + i * q_ls,
+          static_cast<const char*>(k_dev) + i * kv_ls, static_cast<const char*>(v_dev) + i * kv_ls,
+          static_cast<char*>(out_dev) + i * q_ls, stream);
+      if (e != cudaSuccess) return DMC_ERR_CUDA;
+    }
+    return DMC_OK;
+  }
+  const bool pdl = use_pdl(c, first_layer, num_layers);
+  return cuda_status(dmc::decode_launch(L, first_layer, num_layers, c->Gv, c->plan, pdl, q_dev,
+                                        k_dev, v_dev, out_dev, stream));
 }
 
 dmc_status dmc_decode_step_static_scratch(dmc_cache_t c, int32_t layer, const void* q_dev,
@@ -346,10 +388,11 @@ dmc_status dmc_decode_step_static_scratch(dmc_cache_t c, int32_t layer, const vo
   Layout ls = L;
   ls.partials = scratch;
   ls.partial_cap = (int)(floats / state_floats);
-  const bool pdl = use_pdl(c, layer);
+  ls.partials_layer_stride = 0;  // one layer per launch here
+  const bool pdl = use_pdl(c, layer, 1);
   if (c->gqa)
     return cuda_status(dmc::gqa_launch(ls, layer, plan, pdl, q_dev, k_dev, v_dev, out_dev, stream));
-  return cuda_status(dmc::decode_launch(ls, layer, c->Gv, plan, pdl, q_dev, k_dev, v_dev,
+  return cuda_status(dmc::decode_launch(ls, layer, 1, c->Gv, plan, pdl, q_dev, k_dev, v_dev,
                                         out_dev, stream));
 }
 

@@ -56,12 +56,13 @@ enum : int { kFlagAcc = 1, kFlagNaN = 2 };
 
 struct DecodeArgs {
   Layout lay;
-  int layer;
+  int layer0, nlayers;  // layers [layer0, layer0 + nlayers), walked in order
   int Gv;  // virtual heads per KV head: 1, or G when each query head of a group runs alone
-  const char* q;
-  const char* k;
+  const char* q;  // layer layer0 + i at q + i * q_ls bytes: [B][Hq][D]
+  const char* k;  // at k + i * kv_ls: [B][Hkv][D]
   const char* v;
-  char* out;
+  char* out;      // at out + i * q_ls: [B][Hq][D]
+  long long q_ls, kv_ls;
 };
 
 template <typename T, int D>
@@ -200,20 +201,31 @@ dmc_decode_kernel(const DecodeArgs a) {
   const int Gv = a.Gv;
   const int NVH = L.NH * Gv;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  int* ctl = L.ctl + a.layer * 4;
-  const int parity = *reinterpret_cast<volatile int*>(&ctl[0]);
-  const int* len_cur = L.lengths + ((size_t)a.layer * 2 + parity) * L.NH;
-  int* len_nxt = L.lengths + ((size_t)a.layer * 2 + (parity ^ 1)) * L.NH;
-  int* ptab = L.page_table + (size_t)a.layer * L.NH * L.MPH;
-
   unsigned char* ring = smem + (size_t)warp * G_::WARP_BYTES;
   int* wpid = reinterpret_cast<int*>(ring + G_::WRING);
   int* wrws = wpid + kWindow;
   int* misc = reinterpret_cast<int*>(smem + (size_t)kWarps * G_::WARP_BYTES);
   int* U = misc + G_::MISC / 4;
 
+  for (int li = 0; li < a.nlayers; ++li) {
+  const int layer = a.layer0 + li;
+  const char* qL = a.q + (size_t)li * a.q_ls;
+  const char* kL = a.k + (size_t)li * a.kv_ls;
+  const char* vL = a.v + (size_t)li * a.kv_ls;
+  char* outL = a.out + (size_t)li * a.q_ls;
+  int* ctl = L.ctl + layer * 4;
+  const int parity = *reinterpret_cast<volatile int*>(&ctl[0]);
+  const int* len_cur = L.lengths + ((size_t)layer * 2 + parity) * L.NH;
+  int* len_nxt = L.lengths + ((size_t)layer * 2 + (parity ^ 1)) * L.NH;
+  int* ptab = L.page_table + (size_t)layer * L.NH * L.MPH;
+  float* partials = L.partials + (size_t)layer * L.partials_layer_stride;
+  char* pending = L.pending + (size_t)layer * L.NH * 2 * ROW;
+  int* pending_at = L.pending_at + (size_t)layer * L.NH;
+  float* pending_z = L.pending_z + (size_t)layer * L.NH;
+
+  if (li > 0) __syncthreads();  // every warp is done with the previous layer's U and window
   // ---------------------------------------------------------------- prologue
-  scan_units(U, misc, ctl, L.lengths + (size_t)a.layer * 2 * L.NH, L.NH, NVH, Gv);
+  scan_units(U, misc, ctl, L.lengths + (size_t)layer * 2 * L.NH, L.NH, NVH, Gv);
   const long long Utot = U[NVH];
   const int NW = gridDim.x * kWarps;
   const int wid = blockIdx.x * kWarps + warp;
@@ -283,8 +295,10 @@ dmc_decode_kernel(const DecodeArgs a) {
   }
 
   // q, k, v and the slots this launch writes are touched only after this point
-  griddep_wait();
-  griddep_launch_dependents();
+  if (li == 0) {
+    griddep_wait();
+    griddep_launch_dependents();
+  }
 
   if (u0 < u1) {
     // lane i holds the gates of head hb + i
@@ -299,11 +313,11 @@ dmc_decode_kernel(const DecodeArgs a) {
       if (hv < NVH && U[hv] < u1) {
         const int bh = hv / Gv, b = bh / L.Hkv, h = bh % L.Hkv;
         const int len = len_cur[bh];
-        const float x = Elt<T>::to_f(reinterpret_cast<const T*>(a.k)[(size_t)bh * D]);
+        const float x = Elt<T>::to_f(reinterpret_cast<const T*>(kL)[(size_t)bh * D]);
         float qs = 0.f;
         for (int g = 0; g < L.G; ++g)
           qs += Elt<T>::to_f(
-              reinterpret_cast<const T*>(a.q)[((size_t)b * L.Hq + (size_t)h * L.G + g) * D]);
+              reinterpret_cast<const T*>(qL)[((size_t)b * L.Hq + (size_t)h * L.G + g) * D]);
         t_len = len;
         // alpha = round(sigmoid(k[0])) = [k[0] >= 0]; an empty head always appends
         t_flags = ((x >= 0.f && len > 0) ? kFlagAcc : 0) | ((x != x) ? kFlagNaN : 0);
@@ -315,7 +329,7 @@ dmc_decode_kernel(const DecodeArgs a) {
     // the query row of the next head, loaded ahead of its use
     auto q_ptr = [&](int hv) {
       const int bh = hv / Gv, b = bh / L.Hkv, h = bh % L.Hkv, g = hv % Gv;
-      return a.q + ((size_t)b * L.Hq + (size_t)h * L.G + g) * ROW + l8 * 16;
+      return qL + ((size_t)b * L.Hq + (size_t)h * L.G + g) * ROW + l8 * 16;
     };
     uint4 qraw[NCH];
 #pragma unroll
@@ -410,10 +424,10 @@ dmc_decode_kernel(const DecodeArgs a) {
           for (int i = 0; i < EPL; ++i) { rk[i] = 0.f; rv[i] = 0.f; }
           const int W = L.window;
           if (accum) {
-            n_old = L.seglen[((size_t)a.layer * 2 + parity) * L.NH + bh];
+            n_old = L.seglen[((size_t)layer * 2 + parity) * L.NH + bh];
             nwin = min(n_old, W - 1);
-            const char* ring = L.ring + ((size_t)a.layer * L.NH + bh) * W * 2 * ROW;
-            const float* ring_w = L.ring_w + ((size_t)a.layer * L.NH + bh) * W;
+            const char* ring = L.ring + ((size_t)layer * L.NH + bh) * W * 2 * ROW;
+            const float* ring_w = L.ring_w + ((size_t)layer * L.NH + bh) * W;
             for (int e = grp; e < nwin; e += 4) {
               const int pos = (n_old - 1 - e) % W;
               const float w = ring_w[pos];
@@ -464,8 +478,8 @@ dmc_decode_kernel(const DecodeArgs a) {
 #pragma unroll
         for (int c = 0; c < NCH; ++c) {
           float kin[EPC], vin[EPC];
-          CK::unpack(__ldg(reinterpret_cast<const uint4*>(a.k + (size_t)bh * ROW + c * 128 + l8 * 16)), kin);
-          CK::unpack(__ldg(reinterpret_cast<const uint4*>(a.v + (size_t)bh * ROW + c * 128 + l8 * 16)), vin);
+          CK::unpack(__ldg(reinterpret_cast<const uint4*>(kL + (size_t)bh * ROW + c * 128 + l8 * 16)), kin);
+          CK::unpack(__ldg(reinterpret_cast<const uint4*>(vL + (size_t)bh * ROW + c * 128 + l8 * 16)), vin);
           if (c == 0 && l8 == 0) kin[0] = 0.f;  // k[0] <- 0 (Algorithm 1)
           float kn[EPC], vn[EPC];
           if (W > 0) {
@@ -477,7 +491,7 @@ dmc_decode_kernel(const DecodeArgs a) {
             if (vh % Gv == 0) {
               // the new token joins the ring at entry n_old % W (no reader of
               // this launch looks there)
-              char* re = L.ring + ((size_t)a.layer * L.NH + bh) * W * 2 * ROW + (size_t)(n_old % Wm) * 2 * ROW;
+              char* re = L.ring + ((size_t)layer * L.NH + bh) * W * 2 * ROW + (size_t)(n_old % Wm) * 2 * ROW;
               *reinterpret_cast<uint4*>(re + c * 128 + l8 * 16) = CK::pack(kin);
               *reinterpret_cast<uint4*>(re + ROW + c * 128 + l8 * 16) = CK::pack(vin);
             }
@@ -523,7 +537,7 @@ dmc_decode_kernel(const DecodeArgs a) {
           // With grouped queries the other virtual heads of this KV head may
           // still read the old last row and z in this launch: the new row waits
           // in the pending buffer until the launch's last block writes it.
-          char* dst = Gv > 1 ? L.pending + (size_t)bh * 2 * ROW
+          char* dst = Gv > 1 ? pending + (size_t)bh * 2 * ROW
                              : L.pages + (size_t)page * L.page_bytes + (size_t)(slot % kPage) * ROW;
           const size_t vstride = Gv > 1 ? (size_t)ROW : (size_t)kPage * ROW;
           if (ok) {
@@ -535,15 +549,15 @@ dmc_decode_kernel(const DecodeArgs a) {
           }
           if (l8 == 0) {
             if (Gv > 1) {
-              L.pending_at[bh] = ok ? page * kPage + slot % kPage : -1;
-              L.pending_z[bh] = znew;
+              pending_at[bh] = ok ? page * kPage + slot % kPage : -1;
+              pending_z[bh] = znew;
             } else if (ok) {
               L.z[(size_t)page * kPage + slot % kPage] = znew;
             }
             len_nxt[bh] = ok ? slot + 1 : len_old;
             if (W > 0) {
-              L.ring_w[((size_t)a.layer * L.NH + bh) * W + n_old % Wm] = omega;
-              L.seglen[((size_t)a.layer * 2 + (parity ^ 1)) * L.NH + bh] = n_old + 1;
+              L.ring_w[((size_t)layer * L.NH + bh) * W + n_old % Wm] = omega;
+              L.seglen[((size_t)layer * 2 + (parity ^ 1)) * L.NH + bh] = n_old + 1;
             }
             if (flags & kFlagNaN) atomicOr(L.error, DMC_FAULT_NAN_GATE);
           }
@@ -578,7 +592,7 @@ dmc_decode_kernel(const DecodeArgs a) {
           merge_state<EPL>(m, lsum, acc, m2, l2, a2);
         }
         const int b = bh / L.Hkv, h = bh % L.Hkv, g = vh % Gv;
-        T* orow = reinterpret_cast<T*>(a.out) + ((size_t)b * L.Hq + (size_t)h * L.G + g) * D;
+        T* orow = reinterpret_cast<T*>(outL) + ((size_t)b * L.Hq + (size_t)h * L.G + g) * D;
         if (hu0 >= u0 && hend <= u1) {
           // the whole head was in this warp
           if (lane < 8) {
@@ -598,7 +612,7 @@ dmc_decode_kernel(const DecodeArgs a) {
         } else {
           // publish this warp's partial state; the last contributor combines
           const int ps = 2 * wid + (hu0 <= u0 ? 0 : 1);
-          float* pp = L.partials + (size_t)ps * PSTRIDE;
+          float* pp = partials + (size_t)ps * PSTRIDE;
           if (lane == 0) *reinterpret_cast<float2*>(pp) = make_float2(m, lsum);
           // lanes of group g write float4 number g, g + 4, ... of their dims
 #pragma unroll
@@ -625,7 +639,7 @@ dmc_decode_kernel(const DecodeArgs a) {
               for (int cw = wf; cw <= wl; ++cw)
                 ncontrib += range_start(cw, Utot, NW) < range_start(cw + 1, Utot, NW);
             }
-            int* cnt = L.counters + (size_t)a.layer * L.NH * L.G + vh;
+            int* cnt = L.counters + (size_t)layer * L.NH * L.G + vh;
             const int old = atomicAdd(cnt, 1);
             last = (old == ncontrib - 1);
             if (last) *cnt = 0;
@@ -637,14 +651,14 @@ dmc_decode_kernel(const DecodeArgs a) {
               // worker wf + i wrote state 2 (wf + i) + 1 if the head starts
               // inside its range (only possible for i = 0), else 2 (wf + i)
               const int first_off = (hu0 > range_start(wf, Utot, NW)) ? 1 : 0;
-              combine_partials<T, D>(L.partials, wf, first_off, wl - wf + 1, lane, orow);
+              combine_partials<T, D>(partials, wf, first_off, wl - wf + 1, lane, orow);
             } else {
               // fewer units than workers (tiny caches): one unit per non-empty
               // range, so each contributor wrote state 2 cw of its range
               float Mc = -INFINITY, Lc = 0.f;
               for (int cw = wf; cw <= wl; ++cw) {
                 if (range_start(cw, Utot, NW) == range_start(cw + 1, Utot, NW)) continue;
-                Mc = fmaxf(Mc, __ldcg(L.partials + (size_t)(2 * cw) * PSTRIDE));
+                Mc = fmaxf(Mc, __ldcg(partials + (size_t)(2 * cw) * PSTRIDE));
               }
               constexpr int DPL = D / 32;  // output dims per lane
               float Oc[DPL];
@@ -652,7 +666,7 @@ dmc_decode_kernel(const DecodeArgs a) {
               for (int i = 0; i < DPL; ++i) Oc[i] = 0.f;
               for (int cw = wf; cw <= wl; ++cw) {
                 if (range_start(cw, Utot, NW) == range_start(cw + 1, Utot, NW)) continue;
-                const float* cp = L.partials + (size_t)(2 * cw) * PSTRIDE;
+                const float* cp = partials + (size_t)(2 * cw) * PSTRIDE;
                 const float mc = __ldcg(cp);
                 const float cwt = (mc == -INFINITY) ? 0.f : exp2f(mc - Mc);
                 Lc = fmaf(__ldcg(cp + 1), cwt, Lc);
@@ -685,16 +699,16 @@ dmc_decode_kernel(const DecodeArgs a) {
     if (Gv > 1) {
       __threadfence();
       for (int bh = tid; bh < L.NH; bh += kDecodeThreads) {
-        const int at = L.pending_at[bh];
+        const int at = pending_at[bh];
         if (at < 0) continue;
         char* dst = L.pages + (size_t)(at / kPage) * L.page_bytes + (size_t)(at % kPage) * ROW;
-        const char* src = L.pending + (size_t)bh * 2 * ROW;
+        const char* src = pending + (size_t)bh * 2 * ROW;
         for (int i = 0; i < ROW; i += 16) {
           *reinterpret_cast<uint4*>(dst + i) = *reinterpret_cast<const uint4*>(src + i);
           *reinterpret_cast<uint4*>(dst + (size_t)kPage * ROW + i) =
               *reinterpret_cast<const uint4*>(src + ROW + i);
         }
-        L.z[at] = L.pending_z[bh];
+        L.z[at] = pending_z[bh];
       }
       __syncthreads();
     }
@@ -705,6 +719,7 @@ dmc_decode_kernel(const DecodeArgs a) {
       __threadfence();
     }
   }
+  }  // layers
 }
 
 template <typename T, int D>
@@ -770,12 +785,15 @@ static cudaError_t launch_decode(const DecodeArgs& a, const DecodePlan& plan, bo
   return cudaLaunchKernelEx(&cfg, dmc_decode_kernel<T, D, false>, a);
 }
 
-cudaError_t decode_launch(const Layout& L, int layer, int Gv, const DecodePlan& plan, bool pdl,
-                          const void* q, const void* k, const void* v, void* out,
+cudaError_t decode_launch(const Layout& L, int layer0, int nlayers, int Gv, const DecodePlan& plan,
+                          bool pdl, const void* q, const void* k, const void* v, void* out,
                           cudaStream_t stream) {
   DecodeArgs a;
   a.lay = L;
-  a.layer = layer;
+  a.layer0 = layer0;
+  a.nlayers = nlayers;
+  a.q_ls = (long long)L.B * L.Hq * L.row_bytes;
+  a.kv_ls = (long long)L.B * L.Hkv * L.row_bytes;
   a.Gv = Gv;
   a.q = static_cast<const char*>(q);
   a.k = static_cast<const char*>(k);

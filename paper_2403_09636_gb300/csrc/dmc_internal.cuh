@@ -31,13 +31,15 @@ struct Layout {
   int* lengths;            // [L][2][NH]  double-buffered slot counts
   int* ctl;                // [L][4]: parity, finished-block counter
   int* counters;           // [L][NH * G] per (virtual) head combine counters
-  char* pending;           // [NH][2][D]: grouped queries: new last rows awaiting the grid's end
-  int* pending_at;         // [NH]: their slot (page * 32 + row), -1 = none
-  float* pending_z;        // [NH]: their z
+  char* pending;           // [L][NH][2][D]: grouped queries: new last rows awaiting the layer's end
+  int* pending_at;         // [L][NH]: their slot (page * 32 + row), -1 = none
+  float* pending_z;        // [L][NH]: their z
   unsigned long long* pool_top;
   unsigned int* error;
   float* partials;         // [partial_cap][D + 2]: split-K partial softmax states (m, l, acc)
   int partial_cap;
+  long long partials_layer_stride;  // floats between layers' partial states (CUDA-core kernel;
+                                    // 0: one region shared by all layers)
   unsigned char* opens;    // [max_prefill_tokens][Hkv]: token opens a slot
   int* plan;               // [Hkv][plan_stride]: first slot index per prompt chunk
   int plan_stride;

@@ -29,11 +29,11 @@ __device__ __forceinline__ int head_of_unit(const int* U, int n, int u) {
 }
 
 // Exclusive prefix of units per (virtual) head into U[0..nvh], all threads:
-// ceil(len / 32) page units plus one owner unit per head.
+// ceil(len / 32) page units, plus one owner unit per head when owner_units.
 // Reads both slot-count buffers together with the parity word, so the prefix
 // costs one round trip to memory.
 static __device__ void scan_units(int* U, int* wsum, const int* ctl, const int* len_both, int nh,
-                           int nvh, int Gv) {
+                           int nvh, int Gv, int owner_units = 1) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int nthr = blockDim.x, nwarps = nthr >> 5;
   const int per = (nvh + nthr - 1) / nthr;
@@ -42,7 +42,7 @@ static __device__ void scan_units(int* U, int* wsum, const int* ctl, const int* 
   int local = 0;
   for (int i = i0; i < i1; ++i) {
     const int l0 = len_both[i / Gv], l1 = len_both[nh + i / Gv];
-    const int units = ceil_div(parity ? l1 : l0, kPage) + 1;
+    const int units = ceil_div(parity ? l1 : l0, kPage) + owner_units;
     U[i] = units;  // per-head count for now, prefixed below
     local += units;
   }

@@ -114,8 +114,14 @@ class Run:
     them."""
 
     def __init__(self, wl: S.Workload, device, samples, decode_steps=None, cache=None,
-                 check_all_lengths=True, window=0):
+                 check_all_lengths=True, window=0, launch="stream"):
+        """launch: how each decode step runs: "stream" (one dmc_decode_step per
+        layer), "layers" (dmc_decode_step_layers: the layers in two launches,
+        [0, L // 2) and [L // 2, L), or one when L = 1) or "graph" (the
+        per-layer launches of a step captured once in a CUDA graph and
+        replayed with each step's inputs copied into its static buffers)."""
         self.wl = wl
+        self.launch = launch
         self.window = window
         self.samples = list(samples)
         G, d = wl.group, wl.head_dim
@@ -165,11 +171,44 @@ class Run:
         idx = {l: (torch.tensor([b for (_, b, _) in ss], device=device),
                    torch.tensor([h for (_, _, h) in ss], device=device)) for l, ss in by_layer.items()}
         B, Hkv = wl.batch, wl.num_kv_heads
+        NL = wl.num_layers
+        graph = None
+        if launch == "graph" and steps:
+            first = [S.gen_decode(wl, layer, 0, device, p=p) for layer in range(NL)]
+            g_in = [{k_: first[layer][k_].clone() for k_ in ("q", "k", "v")} for layer in range(NL)]
+            g_out = [torch.empty_like(first[layer]["q"]) for layer in range(NL)]
+            torch.cuda.synchronize()
+            graph = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(graph):
+                for layer in range(NL):
+                    x = g_in[layer]
+                    self.cache.decode(layer, x["q"], x["k"], x["v"], g_out[layer])
         for step in range(steps):
-            for layer in range(wl.num_layers):
-                dd = S.gen_decode(wl, layer, step, device, p=p)
-                out = torch.empty_like(dd["q"])
-                self.cache.decode(layer, dd["q"], dd["k"], dd["v"], out)
+            dds = [S.gen_decode(wl, layer, step, device, p=p) for layer in range(NL)]
+            outs = [torch.empty_like(dd["q"]) for dd in dds]
+            if launch == "stream":
+                for layer, dd in enumerate(dds):
+                    self.cache.decode(layer, dd["q"], dd["k"], dd["v"], outs[layer])
+            elif launch == "layers":
+                q = torch.stack([dd["q"] for dd in dds])
+                k = torch.stack([dd["k"] for dd in dds])
+                v = torch.stack([dd["v"] for dd in dds])
+                o = torch.empty_like(q)
+                cut = NL // 2
+                for lo, hi in ((0, cut), (cut, NL)):
+                    if hi > lo:
+                        self.cache.decode_layers(lo, q[lo:hi], k[lo:hi], v[lo:hi], o[lo:hi])
+                outs = list(o.unbind(0))
+            elif launch == "graph":
+                for layer, dd in enumerate(dds):
+                    for k_ in ("q", "k", "v"):
+                        g_in[layer][k_].copy_(dd[k_])
+                graph.replay()
+                outs = [x.clone() for x in g_out]
+            else:
+                raise ValueError(launch)
+            for layer in range(NL):
+                dd, out = dds[layer], outs[layer]
                 if layer in lens_now:
                     exp = expected_step_lengths(lens_now[layer], dd["k"][:, :, 0].float().cpu().numpy())
                     got = self.cache.lengths(layer).cpu().numpy()

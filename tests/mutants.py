@@ -33,13 +33,14 @@ class _Tracked:
     """An oracle HeadCache plus dense copies of its slots, updated in place
     (Algorithm 1 changes only the last slot or appends one)."""
 
-    def __init__(self, d, cap):
+    def __init__(self, d, cap, window=0):
         self.c = R.HeadCache(d)
         self.K = np.zeros((cap, d))
         self.V = np.zeros((cap, d))
+        self.window = window
 
     def update(self, k, v, q0_group):
-        R.update(self.c, k, v, int(R.decision(k[0])), float(R.importance(q0_group)))
+        R.update(self.c, k, v, int(R.decision(k[0])), float(R.importance(q0_group)), self.window)
         n = len(self.c)
         self.K[n - 1] = self.c.K[-1]
         self.V[n - 1] = self.c.V[-1]
@@ -77,10 +78,12 @@ def _heaviest_page(K, V, q):
     return int(np.argmax(mass))
 
 
-def decode_outputs(k_prompt, v_prompt, q0_prompt, k_dec, v_dec, q_dec, modes=MODES + ("exact",)):
+def decode_outputs(k_prompt, v_prompt, q0_prompt, k_dec, v_dec, q_dec, modes=MODES + ("exact",),
+                   window=0):
     """Decode outputs [S, G, d] of one KV head under each mode: the prompt is
     compressed, then every decode token is compressed and its G queries
-    attend (the oracle's run_head with the attention step mutated)."""
+    attend (the oracle's run_head with the attention step mutated; window > 0:
+    the window-grouping approximation)."""
     k_prompt, v_prompt = np.asarray(k_prompt, np.float64), np.asarray(v_prompt, np.float64)
     q0_prompt = np.asarray(q0_prompt, np.float64)
     k_dec, v_dec = np.asarray(k_dec, np.float64), np.asarray(v_dec, np.float64)
@@ -88,7 +91,7 @@ def decode_outputs(k_prompt, v_prompt, q0_prompt, k_dec, v_dec, q_dec, modes=MOD
     T, S = k_prompt.shape[0], k_dec.shape[0]
     d = k_dec.shape[1]
     G = q_dec.shape[1]
-    tr = _Tracked(d, T + S + 1)
+    tr = _Tracked(d, T + S + 1, window)
     for t in range(T):
         tr.update(k_prompt[t], v_prompt[t], q0_prompt[t])
     after_prompt = copy.deepcopy(tr)
@@ -119,3 +122,28 @@ def prompt_outputs(k, v, q, modes=MODES + ("exact",)):
 def separation(got, muts, modes=MODES):
     """max |got - mutant| per mode."""
     return {m: float(np.max(np.abs(np.asarray(got, np.float64) - muts[m]))) for m in modes}
+
+
+def decode_separation(run, tol):
+    """For a harness Run: per sampled head, the GPU decode outputs against each
+    mutant. Returns (worst, failures): worst = smallest distance per mode over
+    the heads where the mode applies (a head of one page has no page to drop),
+    failures = the heads where a mutant lies within `tol`."""
+    worst = {m: np.inf for m in MODES}
+    bad = []
+    for s in run.samples:
+        I = run.inst[s]
+        if not I["out"]:
+            continue
+        got = np.array(I["out"])
+        muts = decode_outputs(I["k_prompt"], I["v_prompt"], I["q0_prompt"], np.array(I["k_dec"]),
+                              np.array(I["v_dec"]), np.array(I["q_dec"]), window=run.window)
+        n_slots = run.final_export[s][3]
+        sep = separation(got, muts)
+        for m in MODES:
+            if m == "droppage" and n_slots <= PAGE:
+                continue
+            worst[m] = min(worst[m], sep[m])
+            if not sep[m] > tol:
+                bad.append(f"{s}: within {sep[m]:.4f} of the '{m}' mutant")
+    return worst, bad
