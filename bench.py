@@ -64,9 +64,16 @@ def parse():
                     help="window-grouping approximation over this many tokens (0: exact DMC)")
     ap.add_argument("--pa-layers", type=int, default=4,
                     help="layers of the prompt-attention measurement (0 skips it)")
-    ap.add_argument("--graph", action="store_true",
-                    help="replay the step's launches from CUDA graphs instead of launching from the host")
-    return ap.parse_args()
+    ap.add_argument("--launch", default="stream", choices=["stream", "graph", "layers"],
+                    help="decode launches: one per layer from the host (stream), the step's "
+                         "launches replayed from CUDA graphs (graph), or one launch per decode "
+                         "step over all layers, dmc_decode_step_layers (layers)")
+    ap.add_argument("--graph", action="store_true", help="same as --launch graph")
+    args = ap.parse_args()
+    if args.graph:
+        args.launch = "graph"
+    args.graph = args.launch == "graph"
+    return args
 
 
 # ------------------------------------------------------------------ helpers
@@ -259,7 +266,8 @@ def workload_config(wl, steps_dec, world, args, l2):
             "seq_len": int(lens.max()) + steps_dec,
             "parallelism": "cpu" if args.impl == "reference" else f"replicas{world}",
             "launch": ("host_threads" if args.impl == "reference" else
-                       "cuda_graph" if args.graph else "stream"),
+                       {"graph": "cuda_graph", "stream": "stream",
+                        "layers": "one launch per step over all layers"}[args.launch]),
             "window": args.window, "l2": l2}
 
 
@@ -372,6 +380,9 @@ def run_ours(args, rank, world, dist):
              for l in range(Lr)] for t in range(steps_dec)]
     h = cache.handle
     pf_fn, dec_fn, reset_fn = L_.dmc_prefill_compress, L_.dmc_decode_step, L_.dmc_cache_reset
+    dec_layers_fn = L_.dmc_decode_step_layers
+    dlay = [(qd[t].data_ptr(), kd[t].data_ptr(), vd[t].data_ptr(), outs.data_ptr())
+            for t in range(steps_dec)]
 
     def prefill_all(sh):
         rc = reset_fn(h, sh)
@@ -383,6 +394,10 @@ def run_ours(args, rank, world, dist):
     def decode_all(sh):
         rc = 0
         for t in range(steps_dec):
+            if args.launch == "layers":
+                a = dlay[t]
+                rc |= dec_layers_fn(h, 0, Lr, a[0], a[1], a[2], a[3], sh)
+                continue
             for l in range(Lr):
                 a = dptr[t][l]
                 rc |= dec_fn(h, l, a[0], a[1], a[2], a[3], sh)
@@ -480,9 +495,11 @@ def run_ours(args, rank, world, dist):
                      "frac": achieved / peak, "traffic": traffic,
                      "algorithmic_bytes_per_launch": per_launch_bytes,
                      "avg_launch_us": avg_launch_s * 1e6,
-                     "timing": "decode-phase CUDA events / launches (launch gaps included)"},
+                     "timing": "decode-phase CUDA events / (decode steps x layers), launch gaps "
+                               "included" + ("; one kernel launch covers all layers of a step"
+                                             if args.launch == "layers" else "")},
         "clocks": clk.summary(),
-        "gpu_launches": K * (2 * Lr + n_dec_launch),
+        "gpu_launches": K * (2 * Lr + (steps_dec if args.launch == "layers" else n_dec_launch)),
     }
 
     # ---- end to end: same step through the C ABI with pinned host buffers
