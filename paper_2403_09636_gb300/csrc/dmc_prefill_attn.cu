@@ -51,7 +51,13 @@ struct PrefillAttnArgs {
   int total_tokens, max_seqlen;
   const float* carry;  // [chunk id][Hkv][2D + 1]
   char* out;           // [total_tokens][Hq][D]
+  int seq_base;        // this launch's first sequence within the call (chunk ids count sequences)
 };
+
+// Sequences per launch: the per-CTA table of work items before each sequence
+// lives in shared memory.
+constexpr int kPaMaxSeqs = 768;
+static_assert(kPaMaxSeqs == 3 * kPaThreads, "three sequences per thread in the item prefix");
 
 // byte offset of 16-byte chunk j (0..15) of row r in a [128 rows][256 B] tile
 // kept as two 128-byte column halves, 128B-swizzled (chunk ^ row % 8)
@@ -148,6 +154,15 @@ __device__ __forceinline__ void fence_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
+// Persistent: each CTA takes query tiles (work items) from a counter in the
+// layer's control words until none is left; the last CTA to finish resets the
+// counter. Items run sequence by sequence and KV head by KV head, so the CTAs
+// at work share a few heads' slot tiles in L2, and each head's tiles from the
+// last (which see the most slots) to the first. TMEM, the mbarriers and their
+// phases live across items, and an item's Q, first K/V tile and per-token
+// inputs are requested while the item before it finishes: Q once the previous
+// diagonal score no longer needs the Q buffer, the rest once its last P V is
+// done.
 template <int G>
 __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const PrefillAttnArgs a) {
   constexpr int D = kPaD;
@@ -157,12 +172,11 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
   extern __shared__ __align__(1024) unsigned char smem[];
   const Layout& L = a.lay;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int tile = blockIdx.x, h = blockIdx.y, s = blockIdx.z;
-  const int bh = (a.first_seq + s) * L.Hkv + h;
 
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kPaMisc);  // [0] S done, [1] O done
   uint32_t* tslot = reinterpret_cast<uint32_t*>(smem + kPaMisc + 16);
   volatile int* s_abort = reinterpret_cast<volatile int*>(smem + kPaMisc + 32);  // a wait gave up
+  volatile int* s_item = reinterpret_cast<volatile int*>(smem + kPaMisc + 40);   // [2] next item
   int* s_len = reinterpret_cast<int*>(smem + kPaMisc + 64);            // [128] slots after token
   float* s_om = reinterpret_cast<float*>(smem + kPaMisc + 64 + 512);   // [128] omega
   float* s_rz = reinterpret_cast<float*>(smem + kPaMisc + 64 + 1024);  // [128] 1 / z after token
@@ -174,100 +188,45 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
   float* s_wz = reinterpret_cast<float*>(smem + kPaMisc + 64 + 3744);  // [4] its last segment's omega sum
   int* s_wm = reinterpret_cast<int*>(smem + kPaMisc + 64 + 3760);      // [4] its last opening token
   int* s_seg = reinterpret_cast<int*>(smem + kPaMisc + 4096);          // [128] first token of the segment, or -1
+  int* s_pref = reinterpret_cast<int*>(smem + kPaMisc + 4608);         // [num_seqs + 1] items before each sequence
 
-  const int t0 = a.cu[s], t1 = a.cu[s + 1];
-  if (!(t0 >= 0 && t0 <= t1 && t1 <= a.total_tokens && t1 - t0 <= a.max_seqlen)) return;
-  const int tok0 = t0 + tile * TT;
-  if (tok0 >= t1) return;
-  const int tokN = min(tok0 + TT, t1);
-  const int c = (tok0 - t0) / kPrefillChunk;
-  const int a0 = t0 + c * kPrefillChunk;  // the chunk holding the tile
-  const int cid = (t0 + c * kPrefillChunk) / kPrefillChunk + s;
-  const int base = L.plan[(size_t)h * L.plan_stride + cid];  // slots before the chunk
-  if (base < 0) return;  // the plan failed (capacity or pool); its fault bit is set
+  int* ctr = L.ctl + a.layer * 4 + 2;  // [0] the next work item, [1] CTAs done
   const int parity = *reinterpret_cast<volatile int*>(&L.ctl[a.layer * 4]);
-  const int len_final = L.lengths[((size_t)a.layer * 2 + parity) * L.NH + bh];
-  const int* ptab = L.page_table + ((size_t)a.layer * L.NH + bh) * L.MPH;
-  const __nv_bfloat16* qg = reinterpret_cast<const __nv_bfloat16*>(a.q);
-  const float* carry = a.carry + ((size_t)cid * L.Hkv + h) * (2 * D + 1);
-
-  // ---- Q and the first K/V tile start streaming before anything else. The
-  // first tile is read up to min(128, len_final) slots: every slot the head
-  // holds has been written, and the staircase mask hides those a row does not
-  // see; tiles after the first are read up to the slots the tile's rows see.
-  const uint32_t sQ = smem_u32(smem + kPaQ);
-  for (int i = tid; i < kPaRows * 16; i += kPaThreads) {
-    const int rr = i >> 4, j = i & 15;
-    const int tt = tok0 + rr / G;
-    const bool ok = tt < tokN;
-    const char* src = a.q + (((size_t)(ok ? tt : tok0) * L.Hq + (size_t)h * G + rr % G) * ROW) + j * 16;
-    cp_async16_zfill(sQ + pa_swz(rr, j), src, ok);
-  }
-  // K (which = 0) or V (which = 1) rows of slot tile jt, slots below hi
-  auto load_tile = [&](int which, int jt, int hi) {
-    const uint32_t dst = smem_u32(smem + (which ? kPaV : kPaK));
-    for (int i = tid; i < kPaSlots * 16; i += kPaThreads) {
-      const int rr = i >> 4, j = i & 15;
-      const int slot = jt * kPaSlots + rr;
-      const bool ok = slot < hi;
-      const int page = ok ? ptab[slot / kPage] : 0;
-      const char* src = L.pages + (size_t)page * L.page_bytes +
-                        (size_t)(ok ? slot % kPage : 0) * ROW + (size_t)which * kPage * ROW + j * 16;
-      cp_async16_zfill(dst + pa_swz(rr, j), src, ok);
-    }
-  };
-  // copy groups, oldest first: Q + K0, V0, then per tile K(j + 1) and V(j + 1)
-  load_tile(0, 0, min(kPaSlots, len_final));
-  cp_async_commit();
-  load_tile(1, 0, min(kPaSlots, len_final));
-  cp_async_commit();
-
-  // ---- per-token decisions, omega, slot counts and 1 / z of the chunk up to
-  // the tile end. z after token i is the omega sum of i's segment so far: from
-  // the segment's opening token, or from the carried sums when no token of the
-  // chunk up to i opens a slot (a segmented prefix sum over the chunk).
-  int incl = 0, seg = 0, lastop = -1;
-  float zs = 0.f;
-  if (tid < kPrefillChunk) {
-    const int tau = a0 + tid;
-    int op = 0;
-    float om = 0.f;
-    if (tau < tokN) {
-      op = L.opens[(size_t)tau * L.Hkv + h];
-      float y = 0.f;
+  // ---- the work items: Hkv x ceil(len / TT) per valid sequence, their
+  // exclusive prefix per sequence (3 sequences per thread, one block scan)
+  {
+    int cnt[3], sum = 0;
 #pragma unroll
-      for (int g = 0; g < G; ++g)
-        y += __bfloat162float(qg[((size_t)tau * L.Hq + (size_t)h * G + g) * D]);
-      om = sigmoidf_(y / (float)G);  // omega = sigmoid(mean of the group's q[0])
+    for (int k = 0; k < 3; ++k) {
+      const int sq = 3 * tid + k;
+      cnt[k] = 0;
+      if (sq < a.num_seqs) {
+        const int t0 = a.cu[sq], t1 = a.cu[sq + 1];
+        if (t0 >= 0 && t0 <= t1 && t1 <= a.total_tokens && t1 - t0 <= a.max_seqlen)
+          cnt[k] = L.Hkv * ((t1 - t0 + TT - 1) / TT);
+      }
+      sum += cnt[k];
     }
-    s_op[tid] = (unsigned char)op;
-    s_om[tid] = om;
-    // within the warp for now: openings up to this token, and the omega sum
-    // back to the last opening (seg: one was found)
-    incl = op;
-    seg = op;
-    zs = om;
-    lastop = op ? tid : -1;  // the last opening token up to this one
+    int incl = sum;
 #pragma unroll
     for (int off = 1; off < 32; off <<= 1) {
       const int o = __shfl_up_sync(0xffffffffu, incl, off);
-      const int so = __shfl_up_sync(0xffffffffu, seg, off);
-      const float zo = __shfl_up_sync(0xffffffffu, zs, off);
-      const int lo = __shfl_up_sync(0xffffffffu, lastop, off);
-      if (lane >= off) {
-        incl += o;
-        if (!seg) zs += zo;
-        seg |= so;
-        lastop = max(lastop, lo);
-      }
+      if (lane >= off) incl += o;
     }
-    if (lane == 31) {
-      s_wc[warp] = incl;
-      s_wf[warp] = seg;
-      s_wz[warp] = zs;
-      s_wm[warp] = lastop;
+    if (lane == 31) s_x[warp] = __int_as_float(incl);
+    __syncthreads();
+    int run = incl - sum;
+    for (int w = 0; w < warp; ++w) run += __float_as_int(s_x[w]);
+#pragma unroll
+    for (int k = 0; k < 3; ++k) {
+      const int sq = 3 * tid + k;
+      if (sq < a.num_seqs) s_pref[sq] = run;
+      run += cnt[k];
     }
+    if (tid == kPaThreads - 1) s_pref[a.num_seqs] = run;  // the last thread's run is the total
+    __syncthreads();
   }
+  const int nitems = s_pref[a.num_seqs];
   if (tid == 0) {
     mbar_init(smem_u32(&bars[0]), 1);
     mbar_init(smem_u32(&bars[1]), 1);
@@ -280,336 +239,511 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
                  "r"(256));
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
   }
-  __syncthreads();
-  if (tid < kPrefillChunk) {
-    int add = base;
-    for (int w = 0; w < warp; ++w) add += s_wc[w];
-    s_len[tid] = incl + add;  // slot count after token a0 + tid
-    for (int w = 0; w < warp; ++w) lastop = max(lastop, s_wm[w]);
-    s_seg[tid] = lastop;
-    if (!seg) {
-      // the segment runs in from earlier warps, or from before the chunk
-      bool found = false;
-      for (int w = warp - 1; w >= 0 && !found; --w) {
-        zs += s_wz[w];
-        found = s_wf[w] != 0;
-      }
-      if (!found) zs += carry[2 * D];  // no opening in the chunk up to here
-    }
-    s_rz[tid] = 1.f / zs;
-  }
-  __syncthreads();
-
-  // ---- thread (r, hf): query row r (token tok0 + r / G, query head h G + r % G),
-  // columns [hf * 64, hf * 64 + 64) of its S and O rows
-  const int r = tid & (kPaRows - 1), hf = tid >> 7;
-  const int tau_r = tok0 + r / G;
-  const bool row_ok = tau_r < tokN;
-  const int nvis = row_ok ? s_len[tau_r - a0] - 1 : 0;  // closed slots this row sees
-  const int nvis_max = s_len[tokN - 1 - a0] - 1;
-  const int vis_hi = min(nvis_max, len_final);          // slots worth loading
-  const int ntiles = (vis_hi + kPaSlots - 1) / kPaSlots;
-
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tslot;
   const uint32_t tS = tmem, tO = tmem + 128;
   const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;  // this warp's TMEM lanes
+  const int hf = tid >> 7;
   const uint32_t col0 = hf * HALF;                                // this thread's first column
   const float qscale = 1.4426950408889634f / sqrtf((float)D);   // log2(e) / sqrt(d_h)
+  uint32_t ph[2] = {0u, 0u};  // phase parity of the next completion of each mbarrier
 
   // Waits for a tensor-core commit. A wait that gives up (mbar_wait sets the
-  // fault bit) raises s_abort; later waits then return at once, and the block
+  // fault bit) raises s_abort; later waits then return at once, and the CTA
   // leaves at the next point where every thread has passed a barrier after
   // the wait: no further MMA is issued, its copies drain, TMEM is freed.
-  auto wait_bar = [&](int which, int ph) {
-    if (*s_abort) return;
-    if (!mbar_wait(smem_u32(&bars[which]), ph, L.error)) *s_abort = 1;
+  auto wait_bar = [&](int which) {
+    if (!*s_abort && !mbar_wait(smem_u32(&bars[which]), ph[which], L.error)) *s_abort = 1;
+    ph[which] ^= 1u;
   };
-  auto leave = [&]() {
-    cp_async_wait<0>();
-    tc_fence_before();
-    __syncthreads();
-    if (warp == 0) {
-      tc_fence_after();
-      asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(256));
+
+  const uint32_t sQ = smem_u32(smem + kPaQ);
+  const __nv_bfloat16* qg = reinterpret_cast<const __nv_bfloat16*>(a.q);
+
+  // One work item: the query tile `tile` (from the sequence's start) of KV
+  // head h of sequence s; base < 0 marks an item with nothing to do (past the
+  // last item, or the plan failed, whose fault bit is then set).
+  struct Item {
+    int s, h, tile, t0, t1, base, len_final;
+  };
+  auto item_of = [&](int item) -> Item {
+    Item w;
+    w.base = -1;
+    w.s = w.h = w.tile = w.t0 = w.t1 = w.len_final = 0;
+    if (item >= nitems) return w;
+    int lo = 0, hi = a.num_seqs - 1;  // the sequence: last s with s_pref[s] <= item
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (s_pref[mid] <= item) lo = mid; else hi = mid - 1;
+    }
+    const int per_head = (s_pref[lo + 1] - s_pref[lo]) / L.Hkv;
+    const int rem = item - s_pref[lo];
+    w.s = lo;
+    w.h = rem / per_head;
+    w.tile = per_head - 1 - rem % per_head;
+    w.t0 = a.cu[lo];
+    w.t1 = a.cu[lo + 1];
+    const int c = w.tile * TT / kPrefillChunk;
+    const int cid = w.t0 / kPrefillChunk + c + a.seq_base + lo;
+    w.base = L.plan[(size_t)w.h * L.plan_stride + cid];  // slots before the chunk
+    w.len_final = L.lengths[((size_t)a.layer * 2 + parity) * L.NH + (a.first_seq + lo) * L.Hkv + w.h];
+    return w;
+  };
+  // Q of an item (not committed: it joins the group of the item's first K tile)
+  auto issue_q = [&](const Item& w) {
+    const int tok0 = w.t0 + w.tile * TT, tokN = min(tok0 + TT, w.t1);
+    for (int i = tid; i < kPaRows * 16; i += kPaThreads) {
+      const int rr = i >> 4, j = i & 15;
+      const int tt = tok0 + rr / G;
+      const bool ok = tt < tokN;
+      const char* src = a.q + (((size_t)(ok ? tt : tok0) * L.Hq + (size_t)w.h * G + rr % G) * ROW) + j * 16;
+      cp_async16_zfill(sQ + pa_swz(rr, j), src, ok);
+    }
+  };
+  // K (which = 0) or V (which = 1) rows of slot tile jt of an item's head, slots below hi
+  auto load_tile_of = [&](const Item& w, int which, int jt, int hi) {
+    const int* ptab = L.page_table + ((size_t)a.layer * L.NH + (a.first_seq + w.s) * L.Hkv + w.h) * L.MPH;
+    const uint32_t dst = smem_u32(smem + (which ? kPaV : kPaK));
+    for (int i = tid; i < kPaSlots * 16; i += kPaThreads) {
+      const int rr = i >> 4, j = i & 15;
+      const int slot = jt * kPaSlots + rr;
+      const bool ok = slot < hi;
+      const int page = ok ? ptab[slot / kPage] : 0;
+      const char* src = L.pages + (size_t)page * L.page_bytes +
+                        (size_t)(ok ? slot % kPage : 0) * ROW + (size_t)which * kPage * ROW + j * 16;
+      cp_async16_zfill(dst + pa_swz(rr, j), src, ok);
+    }
+  };
+  // The first K/V tile, up to min(128, len_final) slots: every slot the head
+  // holds has been written, and the staircase mask hides those a row does not
+  // see. Copy groups, oldest first: Q + K0, V0, then per tile K(j + 1), V(j + 1).
+  auto issue_kv0 = [&](const Item& w) {
+    load_tile_of(w, 0, 0, min(kPaSlots, w.len_final));
+    cp_async_commit();
+    load_tile_of(w, 1, 0, min(kPaSlots, w.len_final));
+    cp_async_commit();
+  };
+  // the per-token inputs of an item's chunk (its decision bytes and the
+  // group's q[0]) for thread tid < 128, into registers
+  int m_op = 0;
+  uint32_t m_q0[(G + 1) / 2];
+  auto load_meta = [&](const Item& w) {
+    const int tok0 = w.t0 + w.tile * TT, tokN = min(tok0 + TT, w.t1);
+    const int tau = w.t0 + (w.tile * TT / kPrefillChunk) * kPrefillChunk + tid;
+    m_op = 0;
+#pragma unroll
+    for (int g = 0; g < (G + 1) / 2; ++g) m_q0[g] = 0u;
+    if (tid < kPrefillChunk && tau < tokN) {
+      m_op = L.opens[(size_t)tau * L.Hkv + w.h];
+      const unsigned short* qs = reinterpret_cast<const unsigned short*>(qg) +
+                                 ((size_t)tau * L.Hq + (size_t)w.h * G) * D;
+#pragma unroll
+      for (int g = 0; g < G; ++g) m_q0[g / 2] |= (uint32_t)qs[(size_t)g * D] << (16 * (g & 1));
     }
   };
 
-  // Per slot tile j, with P kept in tensor memory so that the K buffer frees
-  // as soon as S is computed:
-  //   K(j) landed -> S = Q K^T -> K(j + 1) starts -> softmax, P (bf16) over
-  //   this thread's own S columns -> V(j) landed -> O += P V -> V(j + 1) starts
-  // The copy groups stay in step (one, possibly empty, per K and per V slot),
-  // so "all but the newest group" always means the tile needed next.
-  float m = -INFINITY, l = 0.f;  // l: this thread's half of the row sum
-  for (int jt = 0; jt < ntiles; ++jt) {
-    cp_async_wait<1>();  // Q and K(jt) have landed (this thread's copies)
-    fence_async_smem();
+  if (tid == 0) s_item[0] = atomicAdd(&ctr[0], 1);
+  __syncthreads();
+  int item = s_item[0];
+  Item cur = item_of(item);
+  if (cur.base >= 0) {
+    issue_q(cur);
+    issue_kv0(cur);
+    load_meta(cur);
+  }
+
+  for (int it = 0;; ++it) {
+    if (item >= nitems || *s_abort) break;
+    if (tid == 0) s_item[(it + 1) & 1] = atomicAdd(&ctr[0], 1);  // read after the next barrier
+    if (cur.base < 0) {
+      // the plan failed for this item: nothing was requested for it
+      __syncthreads();
+      item = s_item[(it + 1) & 1];
+      cur = item_of(item);
+      if (cur.base >= 0) {
+        issue_q(cur);
+        issue_kv0(cur);
+        load_meta(cur);
+      }
+      continue;
+    }
+    const int s = cur.s, h = cur.h, t0 = cur.t0, t1 = cur.t1, base = cur.base, len_final = cur.len_final;
+    const int bh = (a.first_seq + s) * L.Hkv + h;
+    const int tok0 = t0 + cur.tile * TT;
+    const int tokN = min(tok0 + TT, t1);
+    const int c = (tok0 - t0) / kPrefillChunk;
+    const int a0 = t0 + c * kPrefillChunk;  // the chunk holding the tile
+    const int cid = t0 / kPrefillChunk + c + a.seq_base + s;
+    const int* ptab = L.page_table + ((size_t)a.layer * L.NH + bh) * L.MPH;
+    const float* carry = a.carry + ((size_t)cid * L.Hkv + h) * (2 * D + 1);
+    auto load_tile = [&](int which, int jt, int hi) { load_tile_of(cur, which, jt, hi); };
+    (void)ptab;
+
+    // ---- per-token decisions, omega, slot counts and 1 / z of the chunk up to
+    // the tile end. z after token i is the omega sum of i's segment so far: from
+    // the segment's opening token, or from the carried sums when no token of the
+    // chunk up to i opens a slot (a segmented prefix sum over the chunk).
+    int incl = 0, seg = 0, lastop = -1;
+    float zs = 0.f;
+    if (tid < kPrefillChunk) {
+      const int tau = a0 + tid;
+      const int op = m_op;  // requested with the item's Q
+      float om = 0.f;
+      if (tau < tokN) {
+        float y = 0.f;
+  #pragma unroll
+        for (int g = 0; g < G; ++g)
+          y += __uint_as_float(((m_q0[g / 2] >> (16 * (g & 1))) & 0xffffu) << 16);
+        om = sigmoidf_(y / (float)G);  // omega = sigmoid(mean of the group's q[0])
+      }
+      s_op[tid] = (unsigned char)op;
+      s_om[tid] = om;
+      // within the warp for now: openings up to this token, and the omega sum
+      // back to the last opening (seg: one was found)
+      incl = op;
+      seg = op;
+      zs = om;
+      lastop = op ? tid : -1;  // the last opening token up to this one
+  #pragma unroll
+      for (int off = 1; off < 32; off <<= 1) {
+        const int o = __shfl_up_sync(0xffffffffu, incl, off);
+        const int so = __shfl_up_sync(0xffffffffu, seg, off);
+        const float zo = __shfl_up_sync(0xffffffffu, zs, off);
+        const int lo = __shfl_up_sync(0xffffffffu, lastop, off);
+        if (lane >= off) {
+          incl += o;
+          if (!seg) zs += zo;
+          seg |= so;
+          lastop = max(lastop, lo);
+        }
+      }
+      if (lane == 31) {
+        s_wc[warp] = incl;
+        s_wf[warp] = seg;
+        s_wz[warp] = zs;
+        s_wm[warp] = lastop;
+      }
+    }
     __syncthreads();
-    if (*s_abort) break;  // uniform: every wait that could raise it is behind the barrier
+    const int item_next = s_item[(it + 1) & 1];
+    const Item nxt = item_of(item_next);  // its loads are long done when its inputs are requested
+    if (tid < kPrefillChunk) {
+      int add = base;
+      for (int w = 0; w < warp; ++w) add += s_wc[w];
+      s_len[tid] = incl + add;  // slot count after token a0 + tid
+      for (int w = 0; w < warp; ++w) lastop = max(lastop, s_wm[w]);
+      s_seg[tid] = lastop;
+      if (!seg) {
+        // the segment runs in from earlier warps, or from before the chunk
+        bool found = false;
+        for (int w = warp - 1; w >= 0 && !found; --w) {
+          zs += s_wz[w];
+          found = s_wf[w] != 0;
+        }
+        if (!found) zs += carry[2 * D];  // no opening in the chunk up to here
+      }
+      s_rz[tid] = 1.f / zs;
+    }
+    __syncthreads();
+  
+    // ---- thread (r, hf): query row r (token tok0 + r / G, query head h G + r % G),
+    // columns [hf * 64, hf * 64 + 64) of its S and O rows
+    const int r = tid & (kPaRows - 1), hf = tid >> 7;
+    const int tau_r = tok0 + r / G;
+    const bool row_ok = tau_r < tokN;
+    const int nvis = row_ok ? s_len[tau_r - a0] - 1 : 0;  // closed slots this row sees
+    const int nvis_max = s_len[tokN - 1 - a0] - 1;
+    const int vis_hi = min(nvis_max, len_final);          // slots worth loading
+    const int ntiles = (vis_hi + kPaSlots - 1) / kPaSlots;
+  
+  
+    // Per slot tile j, with P kept in tensor memory so that the K buffer frees
+    // as soon as S is computed:
+    //   K(j) landed -> S = Q K^T -> K(j + 1) starts -> softmax, P (bf16) over
+    //   this thread's own S columns -> V(j) landed -> O += P V -> V(j + 1) starts
+    // The copy groups stay in step (one, possibly empty, per K and per V slot),
+    // so "all but the newest group" always means the tile needed next.
+    float m = -INFINITY, l = 0.f;  // l: this thread's half of the row sum
+    for (int jt = 0; jt < ntiles; ++jt) {
+      cp_async_wait<1>();  // Q and K(jt) have landed (this thread's copies)
+      fence_async_smem();
+      __syncthreads();
+      if (*s_abort) break;  // uniform: every wait that could raise it is behind the barrier
+      if (tid == 0) {
+        tc_fence_after();
+        const uint32_t kA = sQ, kB = smem_u32(smem + kPaK);
+  #pragma unroll
+        for (int kk = 0; kk < D / 16; ++kk) {
+          const uint32_t off = (kk >> 2) * (kPaRows * 128) + (kk & 3) * 32;
+          pa_mma(tS, pa_desc(kA + off, 16, 1024), pa_desc(kB + off, 16, 1024), pa_idesc(false), kk > 0);
+        }
+        pa_commit(smem_u32(&bars[0]));
+      }
+      wait_bar(0);  // S is in TMEM and the K buffer is free
+      tc_fence_after();
+      if (jt + 1 < ntiles) load_tile(0, jt + 1, vis_hi);
+      cp_async_commit();
+      // ---- online softmax: this thread's half of the row. The running maximum m
+      // moves only when a tile's row maximum exceeds it by more than 8 (P then
+      // stays below 2^8; O and l are rescaled only on a move), in the log2 domain.
+      const int vis_row = min(max(nvis - jt * kPaSlots, 0), kPaSlots);  // visible columns of the row
+      const int vis_me = min(max(vis_row - (int)col0, 0), HALF);         // ... in this half
+      const int vis_warp = __reduce_max_sync(0xffffffffu, vis_me);       // TMEM loads are warp-wide
+      const bool full = __all_sync(0xffffffffu, vis_me == HALF);         // no mask in this warp
+      float mx = -INFINITY;  // of the raw scores
+      for (int c0 = 0; c0 < vis_warp; c0 += 32) {
+        float f[32];
+        pa_ld32(tS + lane_base + col0 + c0, f);
+        if (full) {
+  #pragma unroll
+          for (int i = 0; i < 32; ++i) mx = fmaxf(mx, f[i]);
+        } else {
+  #pragma unroll
+          for (int i = 0; i < 32; ++i)
+            if (c0 + i < vis_me) mx = fmaxf(mx, f[i]);
+        }
+      }
+      s_x[hf * kPaRows + r] = mx * qscale;  // qscale > 0
+      __syncthreads();
+      if (*s_abort) break;
+      const float mt = fmaxf(mx * qscale, s_x[(hf ^ 1) * kPaRows + r]);  // the tile's row maximum
+      const bool grow = mt > m + 8.f;  // false while the row has seen nothing
+      const float mn = grow ? mt : m;
+      const float nmn = -mn;
+      float sum = 0.f;
+      uint32_t pk[HALF / 2];  // P of this half, bf16 pairs
+  #pragma unroll
+      for (int c0 = 0; c0 < HALF; c0 += 32) {
+        float f[32];
+        if (c0 < vis_warp) {
+          pa_ld32(tS + lane_base + col0 + c0, f);
+          if (full) {
+  #pragma unroll
+            for (int i = 0; i < 32; ++i) f[i] = pa_ex2(fmaf(f[i], qscale, nmn));
+          } else {
+  #pragma unroll
+            for (int i = 0; i < 32; ++i) f[i] = (c0 + i < vis_me) ? pa_ex2(fmaf(f[i], qscale, nmn)) : 0.f;
+          }
+        } else {
+  #pragma unroll
+          for (int i = 0; i < 32; ++i) f[i] = 0.f;
+        }
+  #pragma unroll
+        for (int i = 0; i < 32; ++i) sum += f[i];
+  #pragma unroll
+        for (int i = 0; i < 16; ++i) pk[c0 / 2 + i] = Chunk<__nv_bfloat16>::pack2(f[2 * i], f[2 * i + 1]);
+      }
+      // P over the first half of this thread's own S columns: slots col0 + 2i,
+      // col0 + 2i + 1 in column col0 + i (the other half's thread writes its own)
+      {
+        float pf[32];
+  #pragma unroll
+        for (int i = 0; i < 32; ++i) pf[i] = __uint_as_float(pk[i]);
+        pa_st32(tS + lane_base + col0, pf);
+      }
+      // a move of the maximum rescales l and this half of O (rows that saw
+      // nothing yet hold zeros)
+      const bool resc = grow && m != -INFINITY;
+      const float corr = resc ? pa_ex2(m - mn) : 1.f;
+      l = l * corr + sum;
+      if (__any_sync(0xffffffffu, resc)) {
+        for (int c0 = 0; c0 < HALF; c0 += 32) {
+          float f[32];
+          pa_ld32(tO + lane_base + col0 + c0, f);
+  #pragma unroll
+          for (int i = 0; i < 32; ++i) f[i] *= corr;
+          pa_st32(tO + lane_base + col0 + c0, f);
+        }
+      }
+      asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+      m = mn;
+      cp_async_wait<1>();  // V(jt) has landed (K(jt + 1) may still be on its way)
+      fence_async_smem();
+      tc_fence_before();
+      __syncthreads();
+      if (tid == 0) {
+        tc_fence_after();
+        const uint32_t vB = smem_u32(smem + kPaV);
+  #pragma unroll
+        for (int kk = 0; kk < kPaSlots / 16; ++kk) {
+          // slots 16 kk ... from half kk / 4 of the row, 8 packed columns per step
+          const uint32_t aT = tS + (uint32_t)((kk >> 2) * HALF + (kk & 3) * 8);
+          pa_mma_ts(tO, aT, pa_desc(vB + kk * 2048, kPaRows * 128, 1024), pa_idesc(true), jt > 0 || kk > 0);
+        }
+        pa_commit(smem_u32(&bars[1]));
+      }
+      // P V done: O holds this tile, S (P) and the V buffer are free
+      wait_bar(1);
+      tc_fence_after();
+      if (jt + 1 < ntiles) load_tile(1, jt + 1, vis_hi);
+      cp_async_commit();
+    }
+    cp_async_wait<0>();
+    tc_fence_after();
+    __syncthreads();  // every MMA and copy of the loop is over: the K and V buffers are free
+    if (*s_abort) break;
+  
+    // ---- the diagonal state as one more tile. When token i of the chunk
+    // attends, its own slot holds k~ = (c_k [no opening in the chunk up to i] +
+    // sum over j = lo..i of omega_j k_j) / z_i, lo being its segment's first
+    // token in the chunk (c_k: the carried sums), and v~ alike. Its score
+    // q . k~ and its share of O come from the chunk's raw rows:
+    // S_d = Q Kraw^T (with q[0] cleared: the gate is not a feature) summed with
+    // the weights omega_j / z_i, then O += P_d Vraw with
+    // P_d[j] = exp2(score - m) omega_j / z_i over the segment's columns.
+    const int nrows = tokN - a0;
+    if (tid < kPaRows) *reinterpret_cast<__nv_bfloat16*>(smem + kPaQ + pa_swz(tid, 0)) = __float2bfloat16_rn(0.f);
+    {
+      const uint32_t sK = smem_u32(smem + kPaK), sV = smem_u32(smem + kPaV);
+      for (int i = tid; i < kPaRows * 16; i += kPaThreads) {
+        const int rr = i >> 4, j = i & 15;
+        const bool ok = rr < nrows;
+        const size_t src = ((size_t)(a0 + (ok ? rr : 0)) * L.Hkv + h) * ROW + j * 16;
+        cp_async16_zfill(sK + pa_swz(rr, j), a.k + src, ok);
+        cp_async16_zfill(sV + pa_swz(rr, j), a.v + src, ok);
+      }
+      cp_async_commit();
+      cp_async_wait<0>();
+    }
+    fence_async_smem();
+    tc_fence_before();
+    __syncthreads();
     if (tid == 0) {
       tc_fence_after();
-      const uint32_t kA = sQ, kB = smem_u32(smem + kPaK);
-#pragma unroll
+      const uint32_t kB = smem_u32(smem + kPaK);
+  #pragma unroll
       for (int kk = 0; kk < D / 16; ++kk) {
         const uint32_t off = (kk >> 2) * (kPaRows * 128) + (kk & 3) * 32;
-        pa_mma(tS, pa_desc(kA + off, 16, 1024), pa_desc(kB + off, 16, 1024), pa_idesc(false), kk > 0);
+        pa_mma(tS, pa_desc(sQ + off, 16, 1024), pa_desc(kB + off, 16, 1024), pa_idesc(false), kk > 0);
       }
       pa_commit(smem_u32(&bars[0]));
     }
-    wait_bar(0, jt & 1);  // S is in TMEM and the K buffer is free
-    tc_fence_after();
-    if (jt + 1 < ntiles) load_tile(0, jt + 1, vis_hi);
-    cp_async_commit();
-    // ---- online softmax: this thread's half of the row. The running maximum m
-    // moves only when a tile's row maximum exceeds it by more than 8 (P then
-    // stays below 2^8; O and l are rescaled only on a move), in the log2 domain.
-    const int vis_row = min(max(nvis - jt * kPaSlots, 0), kPaSlots);  // visible columns of the row
-    const int vis_me = min(max(vis_row - (int)col0, 0), HALF);         // ... in this half
-    const int vis_warp = __reduce_max_sync(0xffffffffu, vis_me);       // TMEM loads are warp-wide
-    const bool full = __all_sync(0xffffffffu, vis_me == HALF);         // no mask in this warp
-    float mx = -INFINITY;  // of the raw scores
-    for (int c0 = 0; c0 < vis_warp; c0 += 32) {
-      float f[32];
-      pa_ld32(tS + lane_base + col0 + c0, f);
-      if (full) {
-#pragma unroll
-        for (int i = 0; i < 32; ++i) mx = fmaxf(mx, f[i]);
-      } else {
-#pragma unroll
-        for (int i = 0; i < 32; ++i)
-          if (c0 + i < vis_me) mx = fmaxf(mx, f[i]);
+    const int ti = (row_ok ? r / G : 0) + (tok0 - a0);  // the row's token in the chunk
+    const int sg = s_seg[ti];                            // its segment's first token, or -1
+    const int lo = max(sg, 0);
+    const float rz = s_rz[ti];
+    float cdot = 0.f;  // q . c_k over this half's dims, when the segment runs in from before the chunk
+    if (sg < 0) {
+  #pragma unroll
+      for (int jj = 0; jj < 8; ++jj) {
+        const int cj = hf * 8 + jj;
+        float qf[8];
+        Chunk<__nv_bfloat16>::unpack(*reinterpret_cast<const uint4*>(smem + kPaQ + pa_swz(r, cj)), qf);
+  #pragma unroll
+        for (int e = 0; e < 8; ++e) cdot = fmaf(qf[e], carry[cj * 8 + e], cdot);
       }
     }
-    s_x[hf * kPaRows + r] = mx * qscale;  // qscale > 0
-    __syncthreads();
-    if (*s_abort) break;
-    const float mt = fmaxf(mx * qscale, s_x[(hf ^ 1) * kPaRows + r]);  // the tile's row maximum
-    const bool grow = mt > m + 8.f;  // false while the row has seen nothing
-    const float mn = grow ? mt : m;
-    const float nmn = -mn;
-    float sum = 0.f;
-    uint32_t pk[HALF / 2];  // P of this half, bf16 pairs
-#pragma unroll
+    wait_bar(0);  // S_d is in TMEM
+    tc_fence_after();
+    float wsum = 0.f;
+  #pragma unroll
     for (int c0 = 0; c0 < HALF; c0 += 32) {
       float f[32];
-      if (c0 < vis_warp) {
-        pa_ld32(tS + lane_base + col0 + c0, f);
-        if (full) {
-#pragma unroll
-          for (int i = 0; i < 32; ++i) f[i] = pa_ex2(fmaf(f[i], qscale, nmn));
-        } else {
-#pragma unroll
-          for (int i = 0; i < 32; ++i) f[i] = (c0 + i < vis_me) ? pa_ex2(fmaf(f[i], qscale, nmn)) : 0.f;
-        }
-      } else {
-#pragma unroll
-        for (int i = 0; i < 32; ++i) f[i] = 0.f;
+      pa_ld32(tS + lane_base + col0 + c0, f);
+  #pragma unroll
+      for (int i = 0; i < 32; ++i) {
+        const int j = (int)col0 + c0 + i;
+        if (j >= lo && j <= ti) wsum = fmaf(s_om[j], f[i], wsum);
       }
-#pragma unroll
-      for (int i = 0; i < 32; ++i) sum += f[i];
-#pragma unroll
-      for (int i = 0; i < 16; ++i) pk[c0 / 2 + i] = Chunk<__nv_bfloat16>::pack2(f[2 * i], f[2 * i + 1]);
     }
-    // P over the first half of this thread's own S columns: slots col0 + 2i,
-    // col0 + 2i + 1 in column col0 + i (the other half's thread writes its own)
+    s_x[hf * kPaRows + r] = wsum + cdot;
+    __syncthreads();
+    if (*s_abort) break;
+    if (nxt.base >= 0) issue_q(nxt);  // S_d is done and every q . c_k read: the Q buffer is free
+    const float dsc = (s_x[r] + s_x[kPaRows + r]) * rz * qscale;  // the diagonal score (log2 units)
     {
+      const bool grow = dsc > m + 8.f;
+      const float mn = grow ? dsc : m;
+      const bool resc = grow && m != -INFINITY;
+      const float corr = resc ? pa_ex2(m - mn) : 1.f;
+      l *= corr;
+      if (__any_sync(0xffffffffu, resc)) {
+        for (int c0 = 0; c0 < HALF; c0 += 32) {
+          float f[32];
+          pa_ld32(tO + lane_base + col0 + c0, f);
+  #pragma unroll
+          for (int i = 0; i < 32; ++i) f[i] *= corr;
+          pa_st32(tO + lane_base + col0 + c0, f);
+        }
+      }
+      m = mn;
+    }
+    const float pd = pa_ex2(dsc - m);  // the diagonal's weight, below 2^8
+    const float pw = pd * rz;
+    {
+      uint32_t pk[HALF / 2];
+  #pragma unroll
+      for (int c0 = 0; c0 < HALF; c0 += 32) {
+  #pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const int j = (int)col0 + c0 + 2 * i;
+          const float p0 = (j >= lo && j <= ti) ? pw * s_om[j] : 0.f;
+          const float p1 = (j + 1 >= lo && j + 1 <= ti) ? pw * s_om[j + 1] : 0.f;
+          pk[c0 / 2 + i] = Chunk<__nv_bfloat16>::pack2(p0, p1);
+        }
+      }
       float pf[32];
-#pragma unroll
+  #pragma unroll
       for (int i = 0; i < 32; ++i) pf[i] = __uint_as_float(pk[i]);
       pa_st32(tS + lane_base + col0, pf);
     }
-    // a move of the maximum rescales l and this half of O (rows that saw
-    // nothing yet hold zeros)
-    const bool resc = grow && m != -INFINITY;
-    const float corr = resc ? pa_ex2(m - mn) : 1.f;
-    l = l * corr + sum;
-    if (__any_sync(0xffffffffu, resc)) {
-      for (int c0 = 0; c0 < HALF; c0 += 32) {
-        float f[32];
-        pa_ld32(tO + lane_base + col0 + c0, f);
-#pragma unroll
-        for (int i = 0; i < 32; ++i) f[i] *= corr;
-        pa_st32(tO + lane_base + col0 + c0, f);
-      }
-    }
     asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
-    m = mn;
-    cp_async_wait<1>();  // V(jt) has landed (K(jt + 1) may still be on its way)
-    fence_async_smem();
+    s_y[hf * kPaRows + r] = l + (hf == 0 ? pd : 0.f);  // the row sum, the diagonal counted once
     tc_fence_before();
     __syncthreads();
     if (tid == 0) {
       tc_fence_after();
       const uint32_t vB = smem_u32(smem + kPaV);
-#pragma unroll
+  #pragma unroll
       for (int kk = 0; kk < kPaSlots / 16; ++kk) {
-        // slots 16 kk ... from half kk / 4 of the row, 8 packed columns per step
         const uint32_t aT = tS + (uint32_t)((kk >> 2) * HALF + (kk & 3) * 8);
-        pa_mma_ts(tO, aT, pa_desc(vB + kk * 2048, kPaRows * 128, 1024), pa_idesc(true), jt > 0 || kk > 0);
+        pa_mma_ts(tO, aT, pa_desc(vB + kk * 2048, kPaRows * 128, 1024), pa_idesc(true), ntiles > 0 || kk > 0);
       }
       pa_commit(smem_u32(&bars[1]));
     }
-    // P V done: O holds this tile, S (P) and the V buffer are free
-    wait_bar(1, jt & 1);
+    wait_bar(1);
     tc_fence_after();
-    if (jt + 1 < ntiles) load_tile(1, jt + 1, vis_hi);
-    cp_async_commit();
+    if (nxt.base >= 0) {  // the last P V is done: the K and V buffers are free
+      issue_kv0(nxt);
+      load_meta(nxt);
+    }
+    const float inv = 1.f / (s_y[r] + s_y[kPaRows + r]);
+    const float cw = (sg < 0) ? pw : 0.f;  // weight of the carried value sums
+    char* orow = a.out + ((size_t)(row_ok ? tau_r : tok0) * L.Hq + (size_t)h * G + r % G) * ROW;
+    for (int c0 = 0; c0 < HALF; c0 += 32) {
+      float f[32];
+      pa_ld32(tO + lane_base + col0 + c0, f);
+      if (row_ok) {
+  #pragma unroll
+        for (int q4 = 0; q4 < 4; ++q4) {
+          const int cc = col0 + c0 + q4 * 8;
+          float o[8];
+  #pragma unroll
+          for (int e = 0; e < 8; ++e) o[e] = fmaf(cw, carry[D + cc + e], f[q4 * 8 + e]) * inv;
+          *reinterpret_cast<uint4*>(orow + cc * 2) = Chunk<__nv_bfloat16>::pack(o);
+        }
+      }
+    }
+    tc_fence_before();  // this item's TMEM loads are done before the next item's MMAs
+    item = item_next;
+    cur = nxt;
   }
   cp_async_wait<0>();
-  tc_fence_after();
-  __syncthreads();  // every MMA and copy of the loop is over: the K and V buffers are free
-  if (*s_abort) {
-    leave();
-    return;
-  }
-
-  // ---- the diagonal state as one more tile. When token i of the chunk
-  // attends, its own slot holds k~ = (c_k [no opening in the chunk up to i] +
-  // sum over j = lo..i of omega_j k_j) / z_i, lo being its segment's first
-  // token in the chunk (c_k: the carried sums), and v~ alike. Its score
-  // q . k~ and its share of O come from the chunk's raw rows:
-  // S_d = Q Kraw^T (with q[0] cleared: the gate is not a feature) summed with
-  // the weights omega_j / z_i, then O += P_d Vraw with
-  // P_d[j] = exp2(score - m) omega_j / z_i over the segment's columns.
-  const int nrows = tokN - a0;
-  if (tid < kPaRows) *reinterpret_cast<__nv_bfloat16*>(smem + kPaQ + pa_swz(tid, 0)) = __float2bfloat16_rn(0.f);
-  {
-    const uint32_t sK = smem_u32(smem + kPaK), sV = smem_u32(smem + kPaV);
-    for (int i = tid; i < kPaRows * 16; i += kPaThreads) {
-      const int rr = i >> 4, j = i & 15;
-      const bool ok = rr < nrows;
-      const size_t src = ((size_t)(a0 + (ok ? rr : 0)) * L.Hkv + h) * ROW + j * 16;
-      cp_async16_zfill(sK + pa_swz(rr, j), a.k + src, ok);
-      cp_async16_zfill(sV + pa_swz(rr, j), a.v + src, ok);
-    }
-    cp_async_commit();
-    cp_async_wait<0>();
-  }
-  fence_async_smem();
-  tc_fence_before();
-  __syncthreads();
-  if (tid == 0) {
-    tc_fence_after();
-    const uint32_t kB = smem_u32(smem + kPaK);
-#pragma unroll
-    for (int kk = 0; kk < D / 16; ++kk) {
-      const uint32_t off = (kk >> 2) * (kPaRows * 128) + (kk & 3) * 32;
-      pa_mma(tS, pa_desc(sQ + off, 16, 1024), pa_desc(kB + off, 16, 1024), pa_idesc(false), kk > 0);
-    }
-    pa_commit(smem_u32(&bars[0]));
-  }
-  const int ti = (row_ok ? r / G : 0) + (tok0 - a0);  // the row's token in the chunk
-  const int sg = s_seg[ti];                            // its segment's first token, or -1
-  const int lo = max(sg, 0);
-  const float rz = s_rz[ti];
-  float cdot = 0.f;  // q . c_k over this half's dims, when the segment runs in from before the chunk
-  if (sg < 0) {
-#pragma unroll
-    for (int jj = 0; jj < 8; ++jj) {
-      const int cj = hf * 8 + jj;
-      float qf[8];
-      Chunk<__nv_bfloat16>::unpack(*reinterpret_cast<const uint4*>(smem + kPaQ + pa_swz(r, cj)), qf);
-#pragma unroll
-      for (int e = 0; e < 8; ++e) cdot = fmaf(qf[e], carry[cj * 8 + e], cdot);
-    }
-  }
-  wait_bar(0, ntiles & 1);  // S_d is in TMEM
-  tc_fence_after();
-  float wsum = 0.f;
-#pragma unroll
-  for (int c0 = 0; c0 < HALF; c0 += 32) {
-    float f[32];
-    pa_ld32(tS + lane_base + col0 + c0, f);
-#pragma unroll
-    for (int i = 0; i < 32; ++i) {
-      const int j = (int)col0 + c0 + i;
-      if (j >= lo && j <= ti) wsum = fmaf(s_om[j], f[i], wsum);
-    }
-  }
-  s_x[hf * kPaRows + r] = wsum + cdot;
-  __syncthreads();
-  if (*s_abort) {
-    leave();
-    return;
-  }
-  const float dsc = (s_x[r] + s_x[kPaRows + r]) * rz * qscale;  // the diagonal score (log2 units)
-  {
-    const bool grow = dsc > m + 8.f;
-    const float mn = grow ? dsc : m;
-    const bool resc = grow && m != -INFINITY;
-    const float corr = resc ? pa_ex2(m - mn) : 1.f;
-    l *= corr;
-    if (__any_sync(0xffffffffu, resc)) {
-      for (int c0 = 0; c0 < HALF; c0 += 32) {
-        float f[32];
-        pa_ld32(tO + lane_base + col0 + c0, f);
-#pragma unroll
-        for (int i = 0; i < 32; ++i) f[i] *= corr;
-        pa_st32(tO + lane_base + col0 + c0, f);
-      }
-    }
-    m = mn;
-  }
-  const float pd = pa_ex2(dsc - m);  // the diagonal's weight, below 2^8
-  const float pw = pd * rz;
-  {
-    uint32_t pk[HALF / 2];
-#pragma unroll
-    for (int c0 = 0; c0 < HALF; c0 += 32) {
-#pragma unroll
-      for (int i = 0; i < 16; ++i) {
-        const int j = (int)col0 + c0 + 2 * i;
-        const float p0 = (j >= lo && j <= ti) ? pw * s_om[j] : 0.f;
-        const float p1 = (j + 1 >= lo && j + 1 <= ti) ? pw * s_om[j + 1] : 0.f;
-        pk[c0 / 2 + i] = Chunk<__nv_bfloat16>::pack2(p0, p1);
-      }
-    }
-    float pf[32];
-#pragma unroll
-    for (int i = 0; i < 32; ++i) pf[i] = __uint_as_float(pk[i]);
-    pa_st32(tS + lane_base + col0, pf);
-  }
-  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
-  s_y[hf * kPaRows + r] = l + (hf == 0 ? pd : 0.f);  // the row sum, the diagonal counted once
-  tc_fence_before();
-  __syncthreads();
-  if (tid == 0) {
-    tc_fence_after();
-    const uint32_t vB = smem_u32(smem + kPaV);
-#pragma unroll
-    for (int kk = 0; kk < kPaSlots / 16; ++kk) {
-      const uint32_t aT = tS + (uint32_t)((kk >> 2) * HALF + (kk & 3) * 8);
-      pa_mma_ts(tO, aT, pa_desc(vB + kk * 2048, kPaRows * 128, 1024), pa_idesc(true), ntiles > 0 || kk > 0);
-    }
-    pa_commit(smem_u32(&bars[1]));
-  }
-  wait_bar(1, ntiles & 1);
-  tc_fence_after();
-  const float inv = 1.f / (s_y[r] + s_y[kPaRows + r]);
-  const float cw = (sg < 0) ? pw : 0.f;  // weight of the carried value sums
-  char* orow = a.out + ((size_t)(row_ok ? tau_r : tok0) * L.Hq + (size_t)h * G + r % G) * ROW;
-  for (int c0 = 0; c0 < HALF; c0 += 32) {
-    float f[32];
-    pa_ld32(tO + lane_base + col0 + c0, f);
-    if (row_ok) {
-#pragma unroll
-      for (int q4 = 0; q4 < 4; ++q4) {
-        const int cc = col0 + c0 + q4 * 8;
-        float o[8];
-#pragma unroll
-        for (int e = 0; e < 8; ++e) o[e] = fmaf(cw, carry[D + cc + e], f[q4 * 8 + e]) * inv;
-        *reinterpret_cast<uint4*>(orow + cc * 2) = Chunk<__nv_bfloat16>::pack(o);
-      }
-    }
-  }
   tc_fence_before();
   __syncthreads();
   if (warp == 0) {
     tc_fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(256));
+  }
+  if (tid == 0) {  // the last CTA out resets the work counter for the next call
+    __threadfence();
+    if (atomicAdd(&ctr[1], 1) == (int)gridDim.x - 1) {
+      ctr[0] = 0;
+      ctr[1] = 0;
+      __threadfence();
+    }
   }
 }
 
@@ -618,15 +752,31 @@ bool prefill_attn_supported(const Layout& L) {
 }
 
 template <int G>
-static cudaError_t launch_pa(const PrefillAttnArgs& a, cudaStream_t stream) {
+static cudaError_t launch_pa(PrefillAttnArgs a, cudaStream_t stream) {
   cudaError_t e = cudaFuncSetAttribute(dmc_prefill_attn_kernel<G>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, kPaSmem);
+  int dev = 0, sms = 0;
+  if (e == cudaSuccess) e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   if (e != cudaSuccess) return e;
   constexpr int TT = kPaRows / G;
-  const int tiles = (a.max_seqlen + TT - 1) / TT;
-  if (tiles == 0) return cudaSuccess;
-  dmc_prefill_attn_kernel<G><<<dim3(tiles, a.lay.Hkv, a.num_seqs), kPaThreads, kPaSmem, stream>>>(a);
-  return cudaGetLastError();
+  const long long tiles = (a.max_seqlen + TT - 1) / TT;
+  const int num_seqs = a.num_seqs, first_seq = a.first_seq;
+  const int* cu = a.cu;
+  // at most kPaMaxSeqs sequences per launch (the work-item table)
+  for (int s0 = 0; s0 < num_seqs; s0 += kPaMaxSeqs) {
+    a.seq_base = s0;
+    a.num_seqs = min(kPaMaxSeqs, num_seqs - s0);
+    a.first_seq = first_seq + s0;
+    a.cu = cu + s0;
+    const long long items = tiles * a.lay.Hkv * a.num_seqs;  // an upper bound
+    if (items == 0) continue;
+    const int grid = (int)(items < 2LL * sms ? items : 2LL * sms);  // two CTAs per SM (TMEM)
+    dmc_prefill_attn_kernel<G><<<grid, kPaThreads, kPaSmem, stream>>>(a);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
 }
 
 cudaError_t prefill_attn_launch(const Layout& L, int layer, int first_seq, int num_seqs,
