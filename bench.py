@@ -69,6 +69,9 @@ def parse():
                          "launches replayed from CUDA graphs (graph), or one launch per decode "
                          "step over all layers, dmc_decode_step_layers (layers)")
     ap.add_argument("--graph", action="store_true", help="same as --launch graph")
+    ap.add_argument("--layers-leg-steps", type=int, default=2,
+                    help="with --launch stream: also time this many steps with one "
+                         "dmc_decode_step_layers launch per decode step (0 skips it)")
     args = ap.parse_args()
     if args.graph:
         args.launch = "graph"
@@ -501,6 +504,35 @@ def run_ours(args, rank, world, dist):
         "clocks": clk.summary(),
         "gpu_launches": K * (2 * Lr + (steps_dec if args.launch == "layers" else n_dec_launch)),
     }
+
+    # ---- the same step with every decode step in one launch over all layers
+    # (for callers whose inputs of all layers are ready); the headline above
+    # keeps one launch per layer, as a model's layers follow each other
+    if args.launch == "stream" and args.layers_leg_steps > 0:
+        args.launch = "layers"
+        one_step()
+        lev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)]
+               for _ in range(args.layers_leg_steps)]
+        barrier()
+        for e in lev:
+            one_step(e)
+        barrier()
+        args.launch = "stream"
+        st, bits, _ = cache.status()
+        got = torch.stack([cache.lengths(l) for l in range(Lr)])
+        if st != 0 or not torch.equal(got.to(torch.int64), final):
+            raise RuntimeError(f"multi-layer leg: status {st} bits {bits:#x} or slot counts differ")
+        ldec_ms = sum(e[1].elapsed_time(e[2]) for e in lev)
+        ldec_ms = max_over_ranks(dist, [ldec_ms], dev)[0]
+        KL = args.layers_leg_steps
+        l_layer_step_s = ldec_ms / 1e3 / (KL * n_dec_launch)
+        l_achieved = per_launch_bytes / l_layer_step_s / 1e9
+        res["multi_layer"] = {
+            "launch": "one dmc_decode_step_layers launch per decode step over all layers",
+            "steps": KL, "decode_only_tokens_per_s": job_rate(world, KL, Bt * steps_dec, ldec_ms),
+            "avg_layer_step_us": l_layer_step_s * 1e6, "achieved_gbs": l_achieved,
+            "frac_of_peak": l_achieved / peak, "peak": peak,
+            "note": "not the headline: needs every layer's inputs at launch"}
 
     # ---- end to end: same step through the C ABI with pinned host buffers
     if args.pa_layers > 0:

@@ -39,7 +39,14 @@ constexpr int kPaTileBytes = kPaRows * kPaD * 2;  // 32 KB: [128 rows][256 B]
 // dynamic shared memory: Q | K | V | misc, 104 KB: two CTAs per SM (P lives in TMEM)
 constexpr int kPaQ = 0, kPaK = kPaTileBytes, kPaV = 2 * kPaTileBytes;
 constexpr int kPaMisc = 3 * kPaTileBytes;
-constexpr int kPaSmem = kPaMisc + 8192;
+// two copies (by item parity) of a chunk's carried sums, 2D + 1 floats each
+constexpr int kPaCarry = kPaMisc + 8192;
+constexpr int kPaCarryBytes = 1040;
+// the current item's page ids (a head's slots up to 32,768; beyond, the page
+// table is read from global memory)
+constexpr int kPaPages = kPaCarry + 2 * kPaCarryBytes;
+constexpr int kPaMaxPages = 1024;
+constexpr int kPaSmem = kPaPages + kPaMaxPages * 4;  // two CTAs per SM
 
 struct PrefillAttnArgs {
   Layout lay;
@@ -189,6 +196,7 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
   int* s_wm = reinterpret_cast<int*>(smem + kPaMisc + 64 + 3760);      // [4] its last opening token
   int* s_seg = reinterpret_cast<int*>(smem + kPaMisc + 4096);          // [128] first token of the segment, or -1
   int* s_pref = reinterpret_cast<int*>(smem + kPaMisc + 4608);         // [num_seqs + 1] items before each sequence
+  int* s_pages = reinterpret_cast<int*>(smem + kPaPages);              // [kPaMaxPages] the item's page ids
 
   int* ctr = L.ctl + a.layer * 4 + 2;  // [0] the next work item, [1] CTAs done
   const int parity = *reinterpret_cast<volatile int*>(&L.ctl[a.layer * 4]);
@@ -302,28 +310,40 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
       cp_async16_zfill(sQ + pa_swz(rr, j), src, ok);
     }
   };
-  // K (which = 0) or V (which = 1) rows of slot tile jt of an item's head, slots below hi
-  auto load_tile_of = [&](const Item& w, int which, int jt, int hi) {
-    const int* ptab = L.page_table + ((size_t)a.layer * L.NH + (a.first_seq + w.s) * L.Hkv + w.h) * L.MPH;
+  // K (which = 0) or V (which = 1) rows of slot tile jt, slots below hi;
+  // page(p) gives the page id of the head's page p
+  auto load_tile_with = [&](auto page_of, int which, int jt, int hi) {
     const uint32_t dst = smem_u32(smem + (which ? kPaV : kPaK));
     for (int i = tid; i < kPaSlots * 16; i += kPaThreads) {
       const int rr = i >> 4, j = i & 15;
       const int slot = jt * kPaSlots + rr;
       const bool ok = slot < hi;
-      const int page = ok ? ptab[slot / kPage] : 0;
+      const int page = ok ? page_of(slot / kPage) : 0;
       const char* src = L.pages + (size_t)page * L.page_bytes +
                         (size_t)(ok ? slot % kPage : 0) * ROW + (size_t)which * kPage * ROW + j * 16;
       cp_async16_zfill(dst + pa_swz(rr, j), src, ok);
     }
   };
+  auto ptab_of = [&](const Item& w) {
+    return L.page_table + ((size_t)a.layer * L.NH + (a.first_seq + w.s) * L.Hkv + w.h) * L.MPH;
+  };
   // The first K/V tile, up to min(128, len_final) slots: every slot the head
   // holds has been written, and the staircase mask hides those a row does not
   // see. Copy groups, oldest first: Q + K0, V0, then per tile K(j + 1), V(j + 1).
-  auto issue_kv0 = [&](const Item& w) {
-    load_tile_of(w, 0, 0, min(kPaSlots, w.len_final));
+  // pg: the item's first four page ids (the first tile's pages), read early.
+  auto issue_kv0 = [&](const Item& w, const int* pg) {
+    auto page_of = [&](int p) { return pg[p]; };
+    load_tile_with(page_of, 0, 0, min(kPaSlots, w.len_final));
     cp_async_commit();
-    load_tile_of(w, 1, 0, min(kPaSlots, w.len_final));
+    load_tile_with(page_of, 1, 0, min(kPaSlots, w.len_final));
     cp_async_commit();
+  };
+  // the first tile's page ids of an item (the pages the head holds)
+  auto first_pages = [&](const Item& w, int* pg) {
+    const int* pt = ptab_of(w);
+    const int np = ceil_div(w.len_final, kPage);
+#pragma unroll
+    for (int p = 0; p < kPaSlots / kPage; ++p) pg[p] = (w.base >= 0 && p < np) ? pt[p] : 0;
   };
   // the per-token inputs of an item's chunk (its decision bytes and the
   // group's q[0]) for thread tid < 128, into registers
@@ -348,9 +368,11 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
   __syncthreads();
   int item = s_item[0];
   Item cur = item_of(item);
+  int pg_next[kPaSlots / kPage];
   if (cur.base >= 0) {
+    first_pages(cur, pg_next);
     issue_q(cur);
-    issue_kv0(cur);
+    issue_kv0(cur, pg_next);
     load_meta(cur);
   }
 
@@ -363,8 +385,9 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
       item = s_item[(it + 1) & 1];
       cur = item_of(item);
       if (cur.base >= 0) {
+        first_pages(cur, pg_next);
         issue_q(cur);
-        issue_kv0(cur);
+        issue_kv0(cur, pg_next);
         load_meta(cur);
       }
       continue;
@@ -377,9 +400,20 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
     const int a0 = t0 + c * kPrefillChunk;  // the chunk holding the tile
     const int cid = t0 / kPrefillChunk + c + a.seq_base + s;
     const int* ptab = L.page_table + ((size_t)a.layer * L.NH + bh) * L.MPH;
-    const float* carry = a.carry + ((size_t)cid * L.Hkv + h) * (2 * D + 1);
-    auto load_tile = [&](int which, int jt, int hi) { load_tile_of(cur, which, jt, hi); };
-    (void)ptab;
+    // the chunk's carried sums and the head's page ids into shared memory
+    // (visible after the first barrier below; the carry by item parity, since
+    // a thread may start this item while another still reads the previous
+    // item's carry in its epilogue)
+    float* s_carry = reinterpret_cast<float*>(smem + kPaCarry + (it & 1) * kPaCarryBytes);
+    {
+      const float* carry_g = a.carry + ((size_t)cid * L.Hkv + h) * (2 * D + 1);
+      for (int i = tid; i < 2 * D + 1; i += kPaThreads) s_carry[i] = carry_g[i];
+      const int np = min(ceil_div(len_final, kPage), kPaMaxPages);
+      for (int i = tid; i < np; i += kPaThreads) s_pages[i] = ptab[i];
+    }
+    const float* carry = s_carry;
+    auto page_of = [&](int p) { return p < kPaMaxPages ? s_pages[p] : ptab[p]; };
+    auto load_tile = [&](int which, int jt, int hi) { load_tile_with(page_of, which, jt, hi); };
 
     // ---- per-token decisions, omega, slot counts and 1 / z of the chunk up to
     // the tile end. z after token i is the omega sum of i's segment so far: from
@@ -429,6 +463,7 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
     __syncthreads();
     const int item_next = s_item[(it + 1) & 1];
     const Item nxt = item_of(item_next);  // its loads are long done when its inputs are requested
+    first_pages(nxt, pg_next);
     if (tid < kPrefillChunk) {
       int add = base;
       for (int w = 0; w < warp; ++w) add += s_wc[w];
@@ -706,7 +741,7 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
     wait_bar(1);
     tc_fence_after();
     if (nxt.base >= 0) {  // the last P V is done: the K and V buffers are free
-      issue_kv0(nxt);
+      issue_kv0(nxt, pg_next);
       load_meta(nxt);
     }
     const float inv = 1.f / (s_y[r] + s_y[kPaRows + r]);
@@ -755,6 +790,7 @@ template <int G>
 static cudaError_t launch_pa(PrefillAttnArgs a, cudaStream_t stream) {
   cudaError_t e = cudaFuncSetAttribute(dmc_prefill_attn_kernel<G>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, kPaSmem);
+
   int dev = 0, sms = 0;
   if (e == cudaSuccess) e = cudaGetDevice(&dev);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
@@ -771,7 +807,11 @@ static cudaError_t launch_pa(PrefillAttnArgs a, cudaStream_t stream) {
     a.cu = cu + s0;
     const long long items = tiles * a.lay.Hkv * a.num_seqs;  // an upper bound
     if (items == 0) continue;
-    const int grid = (int)(items < 2LL * sms ? items : 2LL * sms);  // two CTAs per SM (TMEM)
+    // two CTAs per SM: their shared memory (2 x 111 KB) and TMEM (2 x 256
+    // columns) fit; a CTA that found no SM slot would only start after the
+    // others and find the work counter empty
+    const long long resident = 2LL * sms;
+    const int grid = (int)(items < resident ? items : resident);
     dmc_prefill_attn_kernel<G><<<grid, kPaThreads, kPaSmem, stream>>>(a);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;

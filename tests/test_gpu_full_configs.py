@@ -40,3 +40,16 @@ def test_full_size_sampled(cuda_dev, name):
     del run, cache
     import torch
     torch.cuda.empty_cache()
+
+
+def test_full_size_multi_layer_launch(cuda_dev):
+    """The bench workload at full size with every decode step as one
+    dmc_decode_step_layers launch over the 32 layers (two calls per step:
+    layers 0-15 and 16-31): every slot count every step, and slots, z and every
+    output of 64 sampled heads against the oracle."""
+    wl = S.WORKLOADS["llama2_7b_4x"]
+    wl, cache = H.full_size_cache(wl, cuda_dev, wl.decode_steps)
+    run = H.Run(wl, cuda_dev, H.random_samples(wl, 64, seed=18), cache=cache, launch="layers")
+    assert run.len_ok, run.len_msgs[:5]
+    bad = run.compare()
+    assert not bad, bad[:10]
