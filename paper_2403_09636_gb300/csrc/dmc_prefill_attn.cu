@@ -42,11 +42,7 @@ constexpr int kPaMisc = 3 * kPaTileBytes;
 // two copies (by item parity) of a chunk's carried sums, 2D + 1 floats each
 constexpr int kPaCarry = kPaMisc + 8192;
 constexpr int kPaCarryBytes = 1040;
-// the current item's page ids (a head's slots up to 32,768; beyond, the page
-// table is read from global memory)
-constexpr int kPaPages = kPaCarry + 2 * kPaCarryBytes;
-constexpr int kPaMaxPages = 1024;
-constexpr int kPaSmem = kPaPages + kPaMaxPages * 4;  // two CTAs per SM
+constexpr int kPaSmem = kPaCarry + 2 * kPaCarryBytes;  // two CTAs per SM
 
 struct PrefillAttnArgs {
   Layout lay;
@@ -108,6 +104,11 @@ __device__ __forceinline__ float pa_ex2(float x) {
   float y;
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
+}
+
+// cp.async of 4 bytes (through L1) into shared memory
+__device__ __forceinline__ void pa_cp_async4(uint32_t dst, const void* src) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(dst), "l"(src) : "memory");
 }
 
 __device__ __forceinline__ void pa_commit(uint32_t bar) {
@@ -196,7 +197,6 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
   int* s_wm = reinterpret_cast<int*>(smem + kPaMisc + 64 + 3760);      // [4] its last opening token
   int* s_seg = reinterpret_cast<int*>(smem + kPaMisc + 4096);          // [128] first token of the segment, or -1
   int* s_pref = reinterpret_cast<int*>(smem + kPaMisc + 4608);         // [num_seqs + 1] items before each sequence
-  int* s_pages = reinterpret_cast<int*>(smem + kPaPages);              // [kPaMaxPages] the item's page ids
 
   int* ctr = L.ctl + a.layer * 4 + 2;  // [0] the next work item, [1] CTAs done
   const int parity = *reinterpret_cast<volatile int*>(&L.ctl[a.layer * 4]);
@@ -299,7 +299,8 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
     w.len_final = L.lengths[((size_t)a.layer * 2 + parity) * L.NH + (a.first_seq + lo) * L.Hkv + w.h];
     return w;
   };
-  // Q of an item (not committed: it joins the group of the item's first K tile)
+  // Q of an item (not committed: it forms a copy group with the item's staged
+  // carried sums)
   auto issue_q = [&](const Item& w) {
     const int tok0 = w.t0 + w.tile * TT, tokN = min(tok0 + TT, w.t1);
     for (int i = tid; i < kPaRows * 16; i += kPaThreads) {
@@ -329,21 +330,23 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
   };
   // The first K/V tile, up to min(128, len_final) slots: every slot the head
   // holds has been written, and the staircase mask hides those a row does not
-  // see. Copy groups, oldest first: Q + K0, V0, then per tile K(j + 1), V(j + 1).
-  // pg: the item's first four page ids (the first tile's pages), read early.
-  auto issue_kv0 = [&](const Item& w, const int* pg) {
-    auto page_of = [&](int p) { return pg[p]; };
+  // see. Copy groups, oldest first: Q (+ carry), K0, V0, then per
+  // tile K(j + 1), V(j + 1).
+  auto issue_kv0 = [&](const Item& w) {
+    const int* pt = ptab_of(w);
+    auto page_of = [&](int p) { return pt[p]; };
     load_tile_with(page_of, 0, 0, min(kPaSlots, w.len_final));
     cp_async_commit();
     load_tile_with(page_of, 1, 0, min(kPaSlots, w.len_final));
     cp_async_commit();
   };
-  // the first tile's page ids of an item (the pages the head holds)
-  auto first_pages = [&](const Item& w, int* pg) {
-    const int* pt = ptab_of(w);
-    const int np = ceil_div(w.len_final, kPage);
-#pragma unroll
-    for (int p = 0; p < kPaSlots / kPage; ++p) pg[p] = (w.base >= 0 && p < np) ? pt[p] : 0;
+  // an item's carried sums, into copy `par` of the carry buffer (requested with
+  // its Q, the two form one copy group)
+  auto issue_carry = [&](const Item& w, int par) {
+    const int cid = w.t0 / kPrefillChunk + w.tile * TT / kPrefillChunk + a.seq_base + w.s;
+    const float* carry_g = a.carry + ((size_t)cid * L.Hkv + w.h) * (2 * D + 1);
+    const uint32_t dc = smem_u32(smem + kPaCarry + par * kPaCarryBytes);
+    for (int i = tid; i < 2 * D + 1; i += kPaThreads) pa_cp_async4(dc + 4 * i, carry_g + i);
   };
   // the per-token inputs of an item's chunk (its decision bytes and the
   // group's q[0]) for thread tid < 128, into registers
@@ -368,11 +371,11 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
   __syncthreads();
   int item = s_item[0];
   Item cur = item_of(item);
-  int pg_next[kPaSlots / kPage];
   if (cur.base >= 0) {
-    first_pages(cur, pg_next);
     issue_q(cur);
-    issue_kv0(cur, pg_next);
+    issue_carry(cur, 0);
+    cp_async_commit();
+    issue_kv0(cur);
     load_meta(cur);
   }
 
@@ -385,9 +388,10 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
       item = s_item[(it + 1) & 1];
       cur = item_of(item);
       if (cur.base >= 0) {
-        first_pages(cur, pg_next);
         issue_q(cur);
-        issue_kv0(cur, pg_next);
+        issue_carry(cur, (it + 1) & 1);
+        cp_async_commit();
+        issue_kv0(cur);
         load_meta(cur);
       }
       continue;
@@ -398,21 +402,16 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
     const int tokN = min(tok0 + TT, t1);
     const int c = (tok0 - t0) / kPrefillChunk;
     const int a0 = t0 + c * kPrefillChunk;  // the chunk holding the tile
-    const int cid = t0 / kPrefillChunk + c + a.seq_base + s;
     const int* ptab = L.page_table + ((size_t)a.layer * L.NH + bh) * L.MPH;
-    // the chunk's carried sums and the head's page ids into shared memory
-    // (visible after the first barrier below; the carry by item parity, since
-    // a thread may start this item while another still reads the previous
-    // item's carry in its epilogue)
-    float* s_carry = reinterpret_cast<float*>(smem + kPaCarry + (it & 1) * kPaCarryBytes);
-    {
-      const float* carry_g = a.carry + ((size_t)cid * L.Hkv + h) * (2 * D + 1);
-      for (int i = tid; i < 2 * D + 1; i += kPaThreads) s_carry[i] = carry_g[i];
-      const int np = min(ceil_div(len_final, kPage), kPaMaxPages);
-      for (int i = tid; i < np; i += kPaThreads) s_pages[i] = ptab[i];
-    }
-    const float* carry = s_carry;
-    auto page_of = [&](int p) { return p < kPaMaxPages ? s_pages[p] : ptab[p]; };
+    // the chunk's carried sums came with this item's Q (copy groups, oldest
+    // first: Q + carry, K0, V0; this
+    // thread's copies of the first have landed here, and the first barrier
+    // below makes all of them visible); the carry is kept by item parity,
+    // since a thread may start this item while another still reads the
+    // previous item's carry in its epilogue
+    cp_async_wait<2>();
+    const float* carry = reinterpret_cast<const float*>(smem + kPaCarry + (it & 1) * kPaCarryBytes);
+    auto page_of = [&](int p) { return ptab[p]; };
     auto load_tile = [&](int which, int jt, int hi) { load_tile_with(page_of, which, jt, hi); };
 
     // ---- per-token decisions, omega, slot counts and 1 / z of the chunk up to
@@ -463,7 +462,6 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
     __syncthreads();
     const int item_next = s_item[(it + 1) & 1];
     const Item nxt = item_of(item_next);  // its loads are long done when its inputs are requested
-    first_pages(nxt, pg_next);
     if (tid < kPrefillChunk) {
       int add = base;
       for (int w = 0; w < warp; ++w) add += s_wc[w];
@@ -686,7 +684,13 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
     s_x[hf * kPaRows + r] = wsum + cdot;
     __syncthreads();
     if (*s_abort) break;
-    if (nxt.base >= 0) issue_q(nxt);  // S_d is done and every q . c_k read: the Q buffer is free
+    if (nxt.base >= 0) {
+      // S_d is done and every q . c_k read: the Q buffer is free, and the
+      // other carry copy (the previous item's) is no longer read
+      issue_q(nxt);
+      issue_carry(nxt, (it + 1) & 1);
+      cp_async_commit();
+    }
     const float dsc = (s_x[r] + s_x[kPaRows + r]) * rz * qscale;  // the diagonal score (log2 units)
     {
       const bool grow = dsc > m + 8.f;
@@ -741,7 +745,7 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
     wait_bar(1);
     tc_fence_after();
     if (nxt.base >= 0) {  // the last P V is done: the K and V buffers are free
-      issue_kv0(nxt, pg_next);
+      issue_kv0(nxt);
       load_meta(nxt);
     }
     const float inv = 1.f / (s_y[r] + s_y[kPaRows + r]);
