@@ -171,8 +171,9 @@ dmc_status dmc_decode_step(dmc_cache_t cache, int32_t layer, const void* q_dev,
  *   q_dev:   [num_layers, batch, num_q_heads, head_dim]
  *   k_dev, v_dev: [num_layers, batch, num_kv_heads, head_dim]
  *   out_dev: [num_layers, batch, num_q_heads, head_dim] (written)
- * Grouped bf16 queries of 2 to 8 per KV head (the tensor-core kernel) are
- * issued as one launch per layer. num_layers = 0 is a no-op. */
+ * Both decode kernels (the CUDA-core one and the tensor-core one for grouped
+ * bf16 queries of 2 to 8 per KV head) walk the layers in one launch.
+ * num_layers = 0 is a no-op. */
 dmc_status dmc_decode_step_layers(dmc_cache_t cache, int32_t first_layer, int32_t num_layers,
                                   const void* q_dev, const void* k_dev, const void* v_dev,
                                   void* out_dev, cudaStream_t stream);

@@ -25,13 +25,14 @@ cudaError_t prefill_attn_launch(const Layout& L, int layer, int first_seq, int n
 cudaError_t decode_static_partials(int device, float** ptr, size_t* floats);
 bool gqa_supported(const Layout& L);
 cudaError_t gqa_setup(const Layout& L, DecodePlan* plan);
-cudaError_t gqa_launch(const Layout& L, int layer, const DecodePlan& plan, bool pdl, const void* q,
+cudaError_t gqa_launch(const Layout& L, int layer0, int nlayers, const DecodePlan& plan, bool pdl, const void* q,
                        const void* k, const void* v, void* out, cudaStream_t stream);
 // Split-K partial states a cache's arena holds: two per worker warp of the
 // decode grid (at most 512 blocks x 8 warps), times the group size for the
 // tensor-core kernel, which keeps one per query.
-constexpr int kMaxWorkerStates = 8192;
-inline size_t partial_states_cap(int G) { return (size_t)kMaxWorkerStates * G; }
+inline size_t partial_states_cap(bool cuda_core, int G) {
+  return cuda_core ? (size_t)kMaxWorkerStates : (size_t)kGqaWorkerStates * G;
+}
 }  // namespace dmc
 
 using dmc::Layout;
@@ -99,14 +100,13 @@ Offsets offsets(const dmc_cache_config* c) {
   o.pool_top = at; at = align_up(at + 8);
   o.error = at; at = align_up(at + 4);
   o.meta_end = at;
-  // The CUDA-core decode kernel (every cache but grouped bf16 queries of 2 to
-  // 8 per KV head, which run on the tensor-core kernel) keeps its split-K
-  // states and pending rows per layer: one launch may walk several layers
-  // whose blocks run at their own pace.
+  // Both decode kernels (the CUDA-core one for every cache but grouped bf16
+  // queries of 2 to 8 per KV head, which run on the tensor-core kernel) keep
+  // their split-K states per layer, and the CUDA-core one its pending rows: one
+  // launch may walk several layers whose blocks run at their own pace.
   const bool cuda_core = !(c->dtype == DMC_BF16 && G >= 2 && G <= 8);
-  const size_t state_layers = cuda_core ? (size_t)c->num_layers : 1;
   o.partials = at;
-  at = align_up(at + state_layers * dmc::partial_states_cap(cuda_core ? 1 : G) * (c->head_dim + 4) * 4);
+  at = align_up(at + (size_t)c->num_layers * dmc::partial_states_cap(cuda_core, G) * (c->head_dim + 4) * 4);
   const size_t pend = (cuda_core && G > 1) ? (size_t)c->num_layers * NH : 0;
   o.pending = at; at = align_up(at + pend * 2 * row);
   o.pending_at = at; at = align_up(at + pend * 4);
@@ -207,8 +207,8 @@ dmc_status dmc_cache_create(const dmc_cache_config* cfg, void* arena_dev, size_t
   L.error = reinterpret_cast<unsigned int*>(base + o.error);
   L.partials = reinterpret_cast<float*>(base + o.partials);
   const bool cuda_core = !(cfg->dtype == DMC_BF16 && L.G >= 2 && L.G <= 8);
-  L.partial_cap = (int)dmc::partial_states_cap(cuda_core ? 1 : L.G);
-  L.partials_layer_stride = cuda_core ? (long long)L.partial_cap * (L.D + 4) : 0;
+  L.partial_cap = (int)dmc::partial_states_cap(cuda_core, L.G);
+  L.partials_layer_stride = (long long)L.partial_cap * (L.D + 4);
   L.opens = reinterpret_cast<unsigned char*>(base + o.opens);
   L.plan = reinterpret_cast<int*>(base + o.plan);
   L.plan_stride = o.plan_stride;
@@ -320,7 +320,7 @@ dmc_status dmc_decode_step(dmc_cache_t c, int32_t layer, const void* q_dev, cons
     return DMC_ERR_INVALID_ARG;
   const bool pdl = use_pdl(c, layer, 1);
   if (c->gqa)
-    return cuda_status(dmc::gqa_launch(L, layer, c->plan, pdl, q_dev, k_dev, v_dev, out_dev, stream));
+    return cuda_status(dmc::gqa_launch(L, layer, 1, c->plan, pdl, q_dev, k_dev, v_dev, out_dev, stream));
   return cuda_status(dmc::decode_launch(L, layer, 1, c->Gv, c->plan, pdl, q_dev, k_dev, v_dev,
                                         out_dev, stream));
 }
@@ -335,21 +335,10 @@ dmc_status dmc_decode_step_layers(dmc_cache_t c, int32_t first_layer, int32_t nu
   if (!aligned16(q_dev) || !aligned16(k_dev) || !aligned16(v_dev) || !aligned16(out_dev) ||
       !q_dev || !k_dev || !v_dev || !out_dev)
     return DMC_ERR_INVALID_ARG;
-  if (c->gqa) {
-    // grouped queries on the tensor cores: one launch per layer
-    const size_t q_ls = (size_t)L.B * L.Hq * L.row_bytes, kv_ls = (size_t)L.B * L.Hkv * L.row_bytes;
-    for (int i = 0; i < num_layers; ++i) {
-      const int layer = first_layer + i;
-      const bool pdl = use_pdl(c, layer, 1);
-      const cudaError_t e = dmc::gqa_launch(
-          L, layer, c->plan, pdl, static_cast<const char*>(q_dev) + i * q_ls,
-          static_cast<const char*>(k_dev) + i * kv_ls, static_cast<const char*>(v_dev) + i * kv_ls,
-          static_cast<char*>(out_dev) + i * q_ls, stream);
-      if (e != cudaSuccess) return DMC_ERR_CUDA;
-    }
-    return DMC_OK;
-  }
   const bool pdl = use_pdl(c, first_layer, num_layers);
+  if (c->gqa)
+    return cuda_status(dmc::gqa_launch(L, first_layer, num_layers, c->plan, pdl, q_dev, k_dev, v_dev,
+                                       out_dev, stream));
   return cuda_status(dmc::decode_launch(L, first_layer, num_layers, c->Gv, c->plan, pdl, q_dev,
                                         k_dev, v_dev, out_dev, stream));
 }
@@ -391,7 +380,7 @@ dmc_status dmc_decode_step_static_scratch(dmc_cache_t c, int32_t layer, const vo
   ls.partials_layer_stride = 0;  // one layer per launch here
   const bool pdl = use_pdl(c, layer, 1);
   if (c->gqa)
-    return cuda_status(dmc::gqa_launch(ls, layer, plan, pdl, q_dev, k_dev, v_dev, out_dev, stream));
+    return cuda_status(dmc::gqa_launch(ls, layer, 1, plan, pdl, q_dev, k_dev, v_dev, out_dev, stream));
   return cuda_status(dmc::decode_launch(ls, layer, 1, c->Gv, plan, pdl, q_dev, k_dev, v_dev,
                                         out_dev, stream));
 }

@@ -19,12 +19,12 @@
 // V) reads without bank conflicts; rows past the head's length are
 // zero-filled. The softmax is online in the log2 domain, per query row.
 //
-// Work split, owner update, split-head combine, double-buffered slot counts and
-// programmatic dependent launch follow the MHA kernel (dmc_decode.cu): units
-// are a head's pages plus one owner unit, split evenly over all warps; the
-// owner applies Algorithm 1 once per KV head, and the new row enters the
-// attention as a one-row tile; a head cut between warps is merged by the last
-// warp to finish it, in worker order.
+// Work split, owner update, split-head combine, double-buffered slot counts,
+// programmatic dependent launch and the walk over several layers in one launch
+// follow the MHA kernel (dmc_decode.cu): units are a head's pages plus one
+// owner unit, split evenly over all warps; the owner applies Algorithm 1 once
+// per KV head, and the new row enters the attention as a one-row tile; a head
+// cut between warps is merged by the last warp to finish it, in worker order.
 #include <math.h>
 
 #include "dmc_internal.cuh"
@@ -37,20 +37,21 @@ constexpr int kGThreads = kGWarps * 32;
 constexpr int kGRing = 4;     // tiles per warp ring (kGRing - 1 in flight)
 constexpr int kTile = 16;     // slots per tile
 constexpr int kGWindow = 64;  // page units per warp window
-constexpr int kGMaxBlocks = 512;
+constexpr int kGMaxBlocks = 256;
 constexpr int kGMaxQueries = 8;
 constexpr int kGHeadWindow = 32;  // KV heads whose gates a warp holds in its lanes
-static_assert(kGMaxBlocks * kGWarps * 2 <= 8192, "partials hold two states per worker");
+static_assert(kGMaxBlocks * kGWarps * 2 <= kGqaWorkerStates, "partials hold two states per worker");
 
 enum : int { kGFlagAcc = 1, kGFlagNaN = 2 };
 
 struct GqaArgs {
   Layout lay;
-  int layer;
-  const char* q;
-  const char* k;
+  int layer0, nlayers;  // layers [layer0, layer0 + nlayers), walked in order
+  const char* q;        // layer layer0 + i at q + i * q_ls bytes: [B][Hq][D]
+  const char* k;        // at k + i * kv_ls: [B][Hkv][D]
   const char* v;
-  char* out;
+  char* out;            // at out + i * q_ls: [B][Hq][D]
+  long long q_ls, kv_ls;
 };
 
 template <int D>
@@ -63,8 +64,9 @@ struct GqaGeom {
   static constexpr int WWIN = 2 * kGWindow * 4;   // page ids, rows to copy
   static constexpr int WARP_BYTES = WRING + WWIN;
   static constexpr int MISC = 64;
+  // two unit prefixes (by layer parity)
   static size_t smem_bytes(int nh) {
-    return (size_t)kGWarps * WARP_BYTES + MISC + (size_t)(nh + 1) * 4;
+    return (size_t)kGWarps * WARP_BYTES + MISC + (size_t)2 * (nh + 1) * 4;
   }
 };
 
@@ -92,25 +94,66 @@ __global__ void __launch_bounds__(kGThreads, 1) dmc_decode_gqa_kernel(const GqaA
   const int NH = L.NH;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int g = lane >> 2, t = lane & 3;  // mma fragment row / column pair
-  int* ctl = L.ctl + a.layer * 4;
-  const int parity = *reinterpret_cast<volatile int*>(&ctl[0]);
-  const int* len_cur = L.lengths + ((size_t)a.layer * 2 + parity) * NH;
-  int* len_nxt = L.lengths + ((size_t)a.layer * 2 + (parity ^ 1)) * NH;
-  int* ptab = L.page_table + (size_t)a.layer * NH * L.MPH;
-
   unsigned char* ring = smem + (size_t)warp * G_::WARP_BYTES;
   int* wpid = reinterpret_cast<int*>(ring + G_::WRING);
   int* wrws = wpid + kGWindow;
   int* misc = reinterpret_cast<int*>(smem + (size_t)kGWarps * G_::WARP_BYTES);
-  int* U = misc + G_::MISC / 4;
+  int* Ubuf = misc + G_::MISC / 4;  // the unit prefixes of layers li (buffer li & 1)
+  volatile int* s_done = misc + 8;  // [2]: warps of the block done with the layer in buffer b
+  volatile int* s_tag = misc + 10;  // [2]: 1 + the index li of the layer whose prefix buffer b holds
+
+  // Walking several layers, a warp goes on to the next layer as soon as its own
+  // part of the current one is done: the block builds the first two layers'
+  // unit prefixes here, and the last of its warps to leave layer li builds
+  // layer li + 2's into the buffer it frees.
+  scan_units(Ubuf, misc, L.ctl + a.layer0 * 4, L.lengths + (size_t)a.layer0 * 2 * NH, NH, NH, 1);
+  if (a.nlayers > 1)
+    scan_units(Ubuf + NH + 1, misc, L.ctl + (a.layer0 + 1) * 4,
+               L.lengths + (size_t)(a.layer0 + 1) * 2 * NH, NH, NH, 1);
+  if (tid == 0) {
+    s_done[0] = s_done[1] = 0;
+    s_tag[0] = 1;
+    s_tag[1] = 2;
+  }
+  __syncthreads();
+
+  for (int li = 0; li < a.nlayers; ++li) {
+  const int layer = a.layer0 + li;
+  const char* qL = a.q + (size_t)li * a.q_ls;
+  const char* kL = a.k + (size_t)li * a.kv_ls;
+  const char* vL = a.v + (size_t)li * a.kv_ls;
+  char* outL = a.out + (size_t)li * a.q_ls;
+  int* ctl = L.ctl + layer * 4;
+  const int parity = *reinterpret_cast<volatile int*>(&ctl[0]);
+  const int* len_cur = L.lengths + ((size_t)layer * 2 + parity) * NH;
+  int* len_nxt = L.lengths + ((size_t)layer * 2 + (parity ^ 1)) * NH;
+  int* ptab = L.page_table + (size_t)layer * NH * L.MPH;
+  float* partials = L.partials + (size_t)layer * L.partials_layer_stride;
+  const int ub = li & 1;
+  int* U = Ubuf + ub * (NH + 1);
 
   // ---------------------------------------------------------------- prologue
-  scan_units(U, misc, ctl, L.lengths + (size_t)a.layer * 2 * NH, NH, NH, 1);
-  const long long Utot = U[NH];
+  bool have_units = true;
+  if (li > 0) {
+    // this layer's unit prefix (built by the block's last warp to leave layer
+    // li - 2); a warp that gives up waiting does no work in the layer
+    const uint64_t w0 = globaltimer_ns();
+    while (s_tag[ub] != li + 1) {
+      __nanosleep(32);
+      if (globaltimer_ns() - w0 > kWaitLimitNs) {
+        if (lane == 0) atomicOr(L.error, DMC_FAULT_WAIT_TIMEOUT);
+        have_units = false;
+        break;
+      }
+    }
+    have_units = __all_sync(0xffffffffu, have_units);
+    __threadfence_block();  // the prefix is read after its tag
+  }
+  const long long Utot = have_units ? U[NH] : 0;
   const int NW = gridDim.x * kGWarps;
   const int wid = blockIdx.x * kGWarps + warp;
-  const int u0 = (int)range_start(wid, Utot, NW);
-  const int u1 = (int)range_start(wid + 1, Utot, NW);
+  const int u0 = have_units ? (int)range_start(wid, Utot, NW) : 0;
+  const int u1 = have_units ? (int)range_start(wid + 1, Utot, NW) : 0;
   const int n = u1 - u0;
   const uint32_t ring_s = smem_u32(ring);
 
@@ -181,8 +224,10 @@ __global__ void __launch_bounds__(kGThreads, 1) dmc_decode_gqa_kernel(const GqaA
   }
 
   // q, k, v and the slots this launch writes are touched only after this point
-  griddep_wait();
-  griddep_launch_dependents();
+  if (li == 0) {
+    griddep_wait();
+    griddep_launch_dependents();
+  }
 
   if (n > 0) {
     // lane i holds the gates of KV head hb + i
@@ -197,11 +242,11 @@ __global__ void __launch_bounds__(kGThreads, 1) dmc_decode_gqa_kernel(const GqaA
       if (hv < NH && U[hv] < u1) {
         const int b = hv / L.Hkv, h = hv % L.Hkv;
         const int len = len_cur[hv];
-        const float x = __bfloat162float(reinterpret_cast<const __nv_bfloat16*>(a.k)[(size_t)hv * D]);
+        const float x = __bfloat162float(reinterpret_cast<const __nv_bfloat16*>(kL)[(size_t)hv * D]);
         float qs = 0.f;
         for (int gg = 0; gg < G; ++gg)
           qs += __bfloat162float(reinterpret_cast<const __nv_bfloat16*>(
-              a.q)[((size_t)b * L.Hq + (size_t)h * G + gg) * D]);
+              qL)[((size_t)b * L.Hq + (size_t)h * G + gg) * D]);
         t_len = len;
         // alpha = round(sigmoid(k[0])) = [k[0] >= 0]; an empty head always appends
         t_flags = ((x >= 0.f && len > 0) ? kGFlagAcc : 0) | ((x != x) ? kGFlagNaN : 0);
@@ -216,7 +261,7 @@ __global__ void __launch_bounds__(kGThreads, 1) dmc_decode_gqa_kernel(const GqaA
     auto load_q = [&](int hv, uint32_t (*qa)[2]) {
       const int b = hv / L.Hkv, h = hv % L.Hkv;
       const uint32_t* qrow = reinterpret_cast<const uint32_t*>(
-          a.q + ((size_t)b * L.Hq + (size_t)h * G + (g < G ? g : 0)) * ROW);
+          qL + ((size_t)b * L.Hq + (size_t)h * G + (g < G ? g : 0)) * ROW);
 #pragma unroll
       for (int kk = 0; kk < KT; ++kk) {
         qa[kk][0] = g < G ? __ldg(qrow + kk * 8 + t) : 0u;
@@ -334,10 +379,10 @@ __global__ void __launch_bounds__(kGThreads, 1) dmc_decode_gqa_kernel(const GqaA
         const float* ring_w = nullptr;
         float zold = 0.f, znew = omega;
         if (W > 0) {
-          ring = L.ring + ((size_t)a.layer * NH + vh) * W * 2 * ROW;
-          ring_w = L.ring_w + ((size_t)a.layer * NH + vh) * W;
+          ring = L.ring + ((size_t)layer * NH + vh) * W * 2 * ROW;
+          ring_w = L.ring_w + ((size_t)layer * NH + vh) * W;
           if (accum) {
-            n_old = L.seglen[((size_t)a.layer * 2 + parity) * NH + vh];
+            n_old = L.seglen[((size_t)layer * 2 + parity) * NH + vh];
             nwin = min(n_old, W - 1);
             for (int e = 0; e < nwin; ++e) znew += ring_w[(n_old - 1 - e) % Wm];
           }
@@ -351,7 +396,7 @@ __global__ void __launch_bounds__(kGThreads, 1) dmc_decode_gqa_kernel(const GqaA
         uint4 nrow = make_uint4(0, 0, 0, 0);
         if (act) {
           float in[8], nw[8];
-          const char* src_in = (is_v ? a.v : a.k) + (size_t)vh * ROW + c * 16;
+          const char* src_in = (is_v ? vL : kL) + (size_t)vh * ROW + c * 16;
           CK::unpack(__ldg(reinterpret_cast<const uint4*>(src_in)), in);
           if (!is_v && c == 0) in[0] = 0.f;  // k[0] <- 0 (Algorithm 1)
           if (W > 0) {
@@ -368,7 +413,7 @@ __global__ void __launch_bounds__(kGThreads, 1) dmc_decode_gqa_kernel(const GqaA
 #pragma unroll
             for (int e = 0; e < 8; ++e) nw[e] /= znew;
             // the new token joins the ring at entry n_old % W
-            char* re = L.ring + ((size_t)a.layer * NH + vh) * W * 2 * ROW + (size_t)(n_old % Wm) * 2 * ROW;
+            char* re = L.ring + ((size_t)layer * NH + vh) * W * 2 * ROW + (size_t)(n_old % Wm) * 2 * ROW;
             *reinterpret_cast<uint4*>(re + (is_v ? ROW : 0) + c * 16) = CK::pack(in);
           } else if (accum) {
             const char* orow = L.pages + (size_t)tgt * L.page_bytes +
@@ -405,8 +450,8 @@ __global__ void __launch_bounds__(kGThreads, 1) dmc_decode_gqa_kernel(const GqaA
           if (ok) L.z[(size_t)page * kPage + slot % kPage] = znew;
           len_nxt[vh] = ok ? slot + 1 : len_old;
           if (W > 0) {
-            L.ring_w[((size_t)a.layer * NH + vh) * W + n_old % Wm] = omega;
-            L.seglen[((size_t)a.layer * 2 + (parity ^ 1)) * NH + vh] = n_old + 1;
+            L.ring_w[((size_t)layer * NH + vh) * W + n_old % Wm] = omega;
+            L.seglen[((size_t)layer * 2 + (parity ^ 1)) * NH + vh] = n_old + 1;
           }
           if (flags & kGFlagNaN) atomicOr(L.error, DMC_FAULT_NAN_GATE);
         }
@@ -431,7 +476,7 @@ __global__ void __launch_bounds__(kGThreads, 1) dmc_decode_gqa_kernel(const GqaA
       if (owner || k == n - 1) {
         // ---- this warp's part of the head is done
         const int b = vh / L.Hkv, h = vh % L.Hkv;
-        __nv_bfloat16* ob = reinterpret_cast<__nv_bfloat16*>(a.out) + ((size_t)b * L.Hq + (size_t)h * G) * D;
+        __nv_bfloat16* ob = reinterpret_cast<__nv_bfloat16*>(outL) + ((size_t)b * L.Hq + (size_t)h * G) * D;
         const int q_lo = 2 * t, q_hi = 2 * t + 1;
         if (hu0 >= u0 && owner) {
           // the whole head was in this warp
@@ -453,7 +498,7 @@ __global__ void __launch_bounds__(kGThreads, 1) dmc_decode_gqa_kernel(const GqaA
           // publish this warp's partial states (one per query); the last
           // contributor combines
           const int ps = 2 * wid + (hu0 <= u0 ? 0 : 1);
-          float* pp = L.partials + (size_t)ps * G * (D + 2);
+          float* pp = partials + (size_t)ps * G * (D + 2);
           if (t == 0 && g < G) {
             pp[(size_t)g * (D + 2)] = m;
             pp[(size_t)g * (D + 2) + 1] = lsum;
@@ -483,7 +528,7 @@ __global__ void __launch_bounds__(kGThreads, 1) dmc_decode_gqa_kernel(const GqaA
               for (int cw = wf; cw <= wl; ++cw)
                 ncontrib += range_start(cw, Utot, NW) < range_start(cw + 1, Utot, NW);
             }
-            int* cnt = L.counters + (size_t)a.layer * NH * G + vh;
+            int* cnt = L.counters + (size_t)layer * NH * G + vh;
             const int old = atomicAdd(cnt, 1);
             last = (old == ncontrib - 1);
             if (last) *cnt = 0;
@@ -499,7 +544,7 @@ __global__ void __launch_bounds__(kGThreads, 1) dmc_decode_gqa_kernel(const GqaA
               const long long cs0 = range_start(cw, Utot, NW);
               if (cs0 == range_start(cw + 1, Utot, NW)) continue;
               const int cs = 2 * cw + (hu0 <= cs0 ? 0 : 1);
-              if (qq < G) Mc = fmaxf(Mc, __ldcg(L.partials + ((size_t)cs * G + qq) * (D + 2)));
+              if (qq < G) Mc = fmaxf(Mc, __ldcg(partials + ((size_t)cs * G + qq) * (D + 2)));
             }
             float Lc = 0.f, Oc[DPQ];
 #pragma unroll
@@ -509,7 +554,7 @@ __global__ void __launch_bounds__(kGThreads, 1) dmc_decode_gqa_kernel(const GqaA
               if (cs0 == range_start(cw + 1, Utot, NW)) continue;
               const int cs = 2 * cw + (hu0 <= cs0 ? 0 : 1);
               if (qq < G) {
-                const float* cp = L.partials + ((size_t)cs * G + qq) * (D + 2);
+                const float* cp = partials + ((size_t)cs * G + qq) * (D + 2);
                 const float mc = __ldcg(cp);
                 const float cwt = (mc == -INFINITY) ? 0.f : exp2f(mc - Mc);
                 Lc = fmaf(__ldcg(cp + 1), cwt, Lc);
@@ -534,16 +579,33 @@ __global__ void __launch_bounds__(kGThreads, 1) dmc_decode_gqa_kernel(const GqaA
   }
   cp_async_wait<0>();
 
-  __syncthreads();
-  if (tid == 0) {
+  // this warp is done with the layer: the grid's last warp out publishes the
+  // new slot counts; the block's last warp out builds the prefix of layer
+  // li + 2 into the buffer the layer used
+  __syncwarp();
+  int last_in_block = 0;
+  if (lane == 0) {
     __threadfence();
     const int old = atomicAdd(&ctl[1], 1);
-    if (old == (int)gridDim.x - 1) {  // last block of the launch: publish the new slot counts
+    if (old == (int)gridDim.x * kGWarps - 1) {
       ctl[1] = 0;
       ctl[0] = parity ^ 1;
       __threadfence();
     }
+    last_in_block = atomicAdd(const_cast<int*>(&s_done[ub]), 1) == kGWarps - 1;
   }
+  last_in_block = __shfl_sync(0xffffffffu, last_in_block, 0);
+  if (last_in_block) {
+    __threadfence_block();  // every warp's reads of the buffer came before its count
+    if (li + 2 < a.nlayers)
+      scan_units_warp(U, L.ctl + (layer + 2) * 4, L.lengths + (size_t)(layer + 2) * 2 * NH, NH);
+    if (lane == 0) {
+      s_done[ub] = 0;
+      __threadfence_block();
+      s_tag[ub] = li + 3;
+    }
+  }
+  }  // layers
 }
 
 template <int D>
@@ -577,6 +639,7 @@ static cudaError_t setup_gqa(const Layout& L, DecodePlan* plan) {
   const long long max_blocks = (max_units + kGWarps - 1) / kGWarps;
   if (max_blocks < plan->grid) plan->grid = (int)max_blocks;
   plan->partial_states = 2 * plan->grid * kGWarps * L.G;
+  if (plan->partial_states > L.partial_cap) return cudaErrorInvalidConfiguration;
   return cudaSuccess;
 }
 
@@ -590,11 +653,14 @@ cudaError_t gqa_setup(const Layout& L, DecodePlan* plan) {
   return cudaErrorInvalidValue;
 }
 
-cudaError_t gqa_launch(const Layout& L, int layer, const DecodePlan& plan, bool pdl, const void* q,
-                       const void* k, const void* v, void* out, cudaStream_t stream) {
+cudaError_t gqa_launch(const Layout& L, int layer0, int nlayers, const DecodePlan& plan, bool pdl,
+                       const void* q, const void* k, const void* v, void* out, cudaStream_t stream) {
   GqaArgs a;
   a.lay = L;
-  a.layer = layer;
+  a.layer0 = layer0;
+  a.nlayers = nlayers;
+  a.q_ls = (long long)L.B * L.Hq * L.row_bytes;
+  a.kv_ls = (long long)L.B * L.Hkv * L.row_bytes;
   a.q = static_cast<const char*>(q);
   a.k = static_cast<const char*>(k);
   a.v = static_cast<const char*>(v);

@@ -70,4 +70,34 @@ static __device__ void scan_units(int* U, int* wsum, const int* ctl, const int* 
   __syncthreads();
 }
 
+// scan_units by one warp, for a single kernel-visible head list (Gv = 1, one
+// owner unit per head): the prefix of a later layer, built while the block's
+// other warps still work.
+static __device__ void scan_units_warp(int* U, const int* ctl, const int* len_both, int nh) {
+  const int lane = threadIdx.x & 31;
+  const int per = (nh + 31) / 32;
+  const int i0 = min(lane * per, nh), i1 = min(i0 + per, nh);
+  const int parity = *reinterpret_cast<const volatile int*>(ctl);
+  int local = 0;
+  for (int i = i0; i < i1; ++i) {
+    const int units = ceil_div(parity ? len_both[nh + i] : len_both[i], kPage) + 1;
+    U[i] = units;
+    local += units;
+  }
+  int incl = local;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const int o = __shfl_up_sync(0xffffffffu, incl, off);
+    if (lane >= off) incl += o;
+  }
+  int run = incl - local;
+  for (int i = i0; i < i1; ++i) {
+    const int units = U[i];
+    U[i] = run;
+    run += units;
+  }
+  if (lane == 31) U[nh] = incl;
+  __syncwarp();
+}
+
 }  // namespace dmc

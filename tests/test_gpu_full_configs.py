@@ -42,14 +42,21 @@ def test_full_size_sampled(cuda_dev, name):
     torch.cuda.empty_cache()
 
 
-def test_full_size_multi_layer_launch(cuda_dev):
-    """The bench workload at full size with every decode step as one
-    dmc_decode_step_layers launch over the 32 layers (two calls per step:
-    layers 0-15 and 16-31): every slot count every step, and slots, z and every
-    output of 64 sampled heads against the oracle."""
-    wl = S.WORKLOADS["llama2_7b_4x"]
+@pytest.mark.parametrize("name", ["llama2_7b_4x", "llama2_70b_gqa_2x"])
+def test_full_size_multi_layer_launch(cuda_dev, name):
+    """The bench workload (MHA, CUDA-core kernel) and the 70B GQA workload
+    (tensor-core kernel) at full size with every decode step as
+    dmc_decode_step_layers launches (two calls per step, each over half the
+    layers): every slot count every step, and slots, z and every output of 64
+    sampled heads against the oracle."""
+    wl = S.WORKLOADS[name]
     wl, cache = H.full_size_cache(wl, cuda_dev, wl.decode_steps)
+    covered = f"{name}: {wl.num_layers} of {S.WORKLOADS[name].num_layers} layers checked"
+    print(f"\n{covered}")
     run = H.Run(wl, cuda_dev, H.random_samples(wl, 64, seed=18), cache=cache, launch="layers")
-    assert run.len_ok, run.len_msgs[:5]
+    assert run.len_ok, (covered, run.len_msgs[:5])
     bad = run.compare()
-    assert not bad, bad[:10]
+    assert not bad, (covered, bad[:10])
+    del run, cache
+    import torch
+    torch.cuda.empty_cache()

@@ -9,10 +9,11 @@ test_gpu_signal.py and must also stay farther than the tolerance from each
 mutant oracle. The multi-layer launch splits the layers over two calls, so a
 first layer other than 0 is covered. Covered: MHA bf16 (several layers, the
 owner warp's pages and splits), fp32 grouped queries on the CUDA-core kernel
-(per-query virtual heads and their pending row), window grouping, grouped
-bf16 queries on the tensor-core kernel (one launch per layer), and the tiny
-fp32 workload. A second test requires the multi-layer launch to give exactly
-the outputs of per-layer launches (the same work split per layer).
+(per-query virtual heads and their pending row), window grouping (MHA and
+grouped queries), grouped bf16 queries on the tensor-core kernel (groups of 4
+at d 128 and 8 at d 64, its own walk over the layers), and the tiny fp32
+workload. A second test requires the multi-layer launch to give exactly the
+outputs of per-layer launches (the same work split per layer).
 """
 import numpy as np
 import pytest
@@ -34,6 +35,8 @@ CASES = [
     (S.Workload("modes_f32_g2", 3, 2, 4, 2, 64, "f32", (60, 200), 10, ("fixed", 3.0), 1.0, seed=402), 0),
     (_sig("modes_window", 3, 2, 4, 4, 128, (60, 400), 10, ("choice", (2.0, 16.0)), 403), 12),
     (_sig("modes_gqa4", 2, 2, 8, 2, 128, (100, 600), 10, ("fixed", 2.0), 404), 0),
+    (_sig("modes_gqa8_d64", 3, 2, 16, 2, 64, (80, 500), 10, ("choice", (1.0, 4.0)), 405), 0),
+    (_sig("modes_gqa2_window", 3, 2, 4, 2, 128, (60, 400), 10, ("choice", (2.0, 16.0)), 406), 12),
     (S.WORKLOADS["tiny_f32"], 0),
 ]
 
@@ -53,7 +56,7 @@ def test_launch_mode_matches_oracle(cuda_dev, case, launch):
     assert not bad, bad[:10]
 
 
-@pytest.mark.parametrize("case", CASES[:3], ids=lambda c: c[0].name)
+@pytest.mark.parametrize("case", CASES[:6], ids=lambda c: c[0].name)
 def test_multi_layer_launch_equals_per_layer_launches(cuda_dev, case):
     wl, window = case
     samples = H.all_samples(wl)
