@@ -651,12 +651,20 @@ def run_e2e(args, wl, cache, prompts, qd, kd, vd, outs, steps_dec, dev, stream, 
     each step copies every layer's prompt (one layer's pinned prompt reused for
     all layers) and every decode step's q/k/v (a pinned ring of `ring`
     distinct steps reused cyclically), and reads every decode output back into
-    a pinned ring. The copies run on one copy stream, as a server prefetches
-    its next inputs: each step's outputs as soon as they are written, the
-    decode inputs two steps ahead (double-buffered), and the next step's
-    prompts in token slices, a few after each decode step's input copy, so
-    that no input copy waits behind a whole prompt; events order every copy
-    against the kernels that use its buffer."""
+    a pinned ring. The copies run as a server prefetches its next inputs, on
+    three copy streams so that no copy the kernels wait for queues behind a
+    bulk one: the decode inputs three steps ahead (three buffers) on one, each
+    step's outputs back as soon as they are written on another (the other
+    direction of the host link), and the next step's prompts, in token slices,
+    on the third, each slice issued after a decode step completes (the host
+    runs ahead of the GPU, so pacing it by the host would send the slices as
+    one burst); events order every copy against the kernels that use its
+    buffer. Each copy is one cudaMemcpyAsync issued
+    through ctypes: the host issues ~40 calls per decode step, and the
+    dispatch cost of tensor copies would leave the GPU waiting for them."""
+    import ctypes
+    import ctypes.util
+
     import torch
 
     Lr = wl.num_layers
@@ -673,11 +681,14 @@ def run_e2e(args, wl, cache, prompts, qd, kd, vd, outs, steps_dec, dev, stream, 
     hqd = qd[:ring].cpu().pin_memory()
     hkd = kd[:ring].cpu().pin_memory()
     hvd = vd[:ring].cpu().pin_memory()
-    gq = [torch.empty_like(qd[0]) for _ in range(2)]
-    gk = [torch.empty_like(kd[0]) for _ in range(2)]
-    gv = [torch.empty_like(vd[0]) for _ in range(2)]
-    go = [torch.empty_like(outs) for _ in range(2)]
+    NBUF = max(1, min(3, steps_dec))  # device buffers of decode inputs and outputs
+    gq = [torch.empty_like(qd[0]) for _ in range(NBUF)]
+    gk = [torch.empty_like(kd[0]) for _ in range(NBUF)]
+    gv = [torch.empty_like(vd[0]) for _ in range(NBUF)]
+    go = [torch.empty_like(outs) for _ in range(NBUF)]
     hout = torch.empty((ring,) + tuple(outs.shape), dtype=outs.dtype).pin_memory()
+    out_bytes = outs.numel() * outs.element_size()
+    assert all(x.is_contiguous() for x in (hqd, hkd, hvd, hout, *gq, *gk, *gv, *go))
     h, sh = cache.handle, stream.cuda_stream
     tot, mx, ns = int(cu[-1]), pr0["max_seqlen"], cu.numel() - 1
     h2d = Lr * (hq0.numel() * hq0.element_size() + hk.numel() * hk.element_size() +
@@ -686,47 +697,65 @@ def run_e2e(args, wl, cache, prompts, qd, kd, vd, outs, steps_dec, dev, stream, 
         gv[0].numel() * gv[0].element_size())
     d2h = steps_dec * outs.numel() * outs.element_size()
 
-    cs_io = torch.cuda.Stream(dev)  # every copy, in the order the kernels need them
+    rt = ctypes.CDLL(ctypes.util.find_library("cudart") or "libcudart.so")
+    rt.cudaMemcpyAsync.argtypes = [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_size_t, ctypes.c_int,
+                                   ctypes.c_void_p]
+    rt.cudaMemcpyAsync.restype = ctypes.c_int
+    H2D, D2H = 1, 2  # cudaMemcpyHostToDevice, cudaMemcpyDeviceToHost
+
+    def memcpy(dst, src, nbytes, kind, cs):
+        if rt.cudaMemcpyAsync(dst, src, nbytes, kind, cs.cuda_stream) != 0:
+            raise RuntimeError("cudaMemcpyAsync failed")
+
+    cs_in = torch.cuda.Stream(dev)   # decode inputs
+    cs_out = torch.cuda.Stream(dev)  # decode outputs back to the host
+    cs_pr = torch.cuda.Stream(dev)   # prompts
     ev = lambda: torch.cuda.Event()
     ev_pr = [ev() for _ in range(Lr)]   # prompt of layer l landed
     ev_pf = ev()                        # this step's prefill is done with the prompt buffers
-    ev_in = [ev() for _ in range(2)]    # decode inputs of buffer b landed
-    ev_done = [ev() for _ in range(2)]  # decodes of buffer b done (inputs free, outputs ready)
-    ev_d2h = [ev() for _ in range(2)]   # outputs of buffer b read back
+    ev_in = [ev() for _ in range(NBUF)]    # decode inputs of buffer b landed
+    ev_done = [ev() for _ in range(NBUF)]  # decodes of buffer b done (inputs free, outputs ready)
+    ev_d2h = [ev() for _ in range(NBUF)]   # outputs of buffer b read back
     # the next step's prompts go in NC token slices, a few after each decode
     # step's input copy, so that no input copy waits behind a whole prompt
     CPL = 16                            # slices per layer
     NC = Lr * CPL
     bounds = [tot * j // CPL for j in range(CPL + 1)]
 
-    def copy_prompt_slice(k):  # on cs_io
+    # token-major rows: a slice of tokens [a, b) is one contiguous range
+    prow = [(x.stride(0) * x.element_size(), hx.data_ptr(), [d.data_ptr() for d in dl])
+            for x, hx, dl in ((hq0, hq0, dq0), (hk, hk, dk), (hv, hv, dv))]
+    for (rb, _, dl), x in zip(prow, (dq0, dk, dv)):
+        assert all(d.is_contiguous() and d.stride(0) * d.element_size() == rb for d in x)
+    assert hq0.is_contiguous() and hk.is_contiguous() and hv.is_contiguous()
+
+    def copy_prompt_slice(k):  # on cs_pr
         l, j = divmod(k, CPL)
         a, b = bounds[j], bounds[j + 1]
-        dq0[l][a:b].copy_(hq0[a:b], non_blocking=True)
-        dk[l][a:b].copy_(hk[a:b], non_blocking=True)
-        dv[l][a:b].copy_(hv[a:b], non_blocking=True)
+        for rb, hp, dl in prow:
+            memcpy(dl[l] + a * rb, hp + a * rb, (b - a) * rb, H2D, cs_pr)
         if j == CPL - 1:
-            ev_pr[l].record(cs_io)
+            ev_pr[l].record(cs_pr)
 
     def copy_prompts():  # all at once (the first step's)
-        with torch.cuda.stream(cs_io):
-            for k in range(NC):
-                copy_prompt_slice(k)
+        for k in range(NC):
+            copy_prompt_slice(k)
+
+    dec_bytes = [x[0].numel() * x[0].element_size() for x in (hqd, hkd, hvd)]
 
     def copy_inputs(t, b):
-        with torch.cuda.stream(cs_io):
-            cs_io.wait_event(ev_done[b])
-            gq[b].copy_(hqd[t % ring], non_blocking=True)
-            gk[b].copy_(hkd[t % ring], non_blocking=True)
-            gv[b].copy_(hvd[t % ring], non_blocking=True)
-            ev_in[b].record(cs_io)
+        cs_in.wait_event(ev_done[b])
+        for hx, gx, nb in zip((hqd, hkd, hvd), (gq, gk, gv), dec_bytes):
+            memcpy(gx[b].data_ptr(), hx[t % ring].data_ptr(), nb, H2D, cs_in)
+        ev_in[b].record(cs_in)
 
     def run(nsteps):
         # the first step's prompts and first two decode steps' inputs
-        cs_io.wait_stream(stream)
+        for cs in (cs_in, cs_out, cs_pr):
+            cs.wait_stream(stream)
         copy_prompts()
-        copy_inputs(0, 0)
-        copy_inputs(1 % steps_dec, 1)
+        for j in range(NBUF):
+            copy_inputs(j % steps_dec, j)
         for i in range(nsteps):
             rc = L_.dmc_cache_reset(h, sh)
             for l in range(Lr):
@@ -737,31 +766,33 @@ def run_e2e(args, wl, cache, prompts, qd, kd, vd, outs, steps_dec, dev, stream, 
             ev_pf.record(stream)
             nxt = i + 1 < nsteps  # the next step's prompts stream during this step's decode
             if nxt:
-                with torch.cuda.stream(cs_io):
-                    cs_io.wait_event(ev_pf)
+                cs_pr.wait_event(ev_pf)
             for t in range(steps_dec):
-                b = t & 1
+                b = t % NBUF
                 stream.wait_event(ev_in[b])
-                stream.wait_event(ev_d2h[b])  # outputs of two steps ago are read back
+                stream.wait_event(ev_d2h[b])  # outputs of NBUF steps ago are read back
                 for l in range(Lr):
                     rc |= L_.dmc_decode_step(h, l, gq[b][l].data_ptr(), gk[b][l].data_ptr(),
                                              gv[b][l].data_ptr(), go[b][l].data_ptr(), sh)
                 ev_done[b].record(stream)
-                with torch.cuda.stream(cs_io):
-                    cs_io.wait_event(ev_done[b])
-                    hout[t % ring].copy_(go[b], non_blocking=True)
-                    ev_d2h[b].record(cs_io)
-                last = i + 1 == nsteps and t + 2 >= steps_dec
+                cs_out.wait_event(ev_done[b])
+                memcpy(hout[t % ring].data_ptr(), go[b].data_ptr(), out_bytes, D2H, cs_out)
+                ev_d2h[b].record(cs_out)
+                last = i + 1 == nsteps and t + NBUF >= steps_dec
                 if not last:
-                    # two steps ahead (at the end of a step, the next step's first two)
-                    copy_inputs((t + 2) % steps_dec, b)
+                    # NBUF steps ahead (at the end of a step, the next step's first ones)
+                    copy_inputs((t + NBUF) % steps_dec, b)
                 if nxt:
-                    with torch.cuda.stream(cs_io):
-                        for k in range(t * NC // steps_dec, (t + 1) * NC // steps_dec):
-                            copy_prompt_slice(k)
+                    # paced on the GPU (after this decode step), so that the
+                    # slices do not reach the copy engine as one burst that
+                    # the next decode inputs would queue behind
+                    cs_pr.wait_event(ev_done[b])
+                    for k in range(t * NC // steps_dec, (t + 1) * NC // steps_dec):
+                        copy_prompt_slice(k)
             if rc:
                 raise RuntimeError(f"launch failed: {rc}")
-        stream.wait_stream(cs_io)
+        for cs in (cs_in, cs_out, cs_pr):
+            stream.wait_stream(cs)
 
     run(max(1, args.warmup))
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -778,8 +809,8 @@ def run_e2e(args, wl, cache, prompts, qd, kd, vd, outs, steps_dec, dev, stream, 
             "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
             "note": f"pinned host inputs: one layer's prompt reused for all {Lr} layers, a ring of "
                     f"{ring} decode steps reused cyclically; every attention output is read back into a "
-                    f"pinned ring of {ring} steps; copies on a side stream overlap the kernels "
-                    "(decode inputs two steps ahead; the next step's prompts in slices between them)"}
+                    f"pinned ring of {ring} steps; copies on three side streams overlap the kernels "
+                    "(decode inputs three steps ahead, outputs back, the next step's prompts in slices)"}
 
 
 def main():
