@@ -313,16 +313,32 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
   };
   // K (which = 0) or V (which = 1) rows of slot tile jt, slots below hi;
   // page(p) gives the page id of the head's page p
-  auto load_tile_with = [&](auto page_of, int which, int jt, int hi) {
+  // Slot tile jt of a head into the K (which = 0) or V buffer, slots past hi
+  // zero-filled; pg[q] is the page of the tile's slots [32 q, 32 q + 32). A
+  // thread copies 16 bytes of rows tid / 16 + 16 k, k = 0..7, which lie in
+  // page k / 2 of the tile (tid / 16 < 16), so the page ids are read by
+  // compile-time index.
+  static_assert(kPaThreads == 256 && kPaSlots == 4 * kPage, "row k of a thread lies in page k / 2");
+  auto load_tile_pg = [&](const int* pg, int which, int jt, int hi) {
     const uint32_t dst = smem_u32(smem + (which ? kPaV : kPaK));
-    for (int i = tid; i < kPaSlots * 16; i += kPaThreads) {
-      const int rr = i >> 4, j = i & 15;
+    const int j = tid & 15;
+#pragma unroll
+    for (int k = 0; k < kPaSlots * 16 / kPaThreads; ++k) {
+      const int rr = (tid >> 4) + 16 * k;
       const int slot = jt * kPaSlots + rr;
       const bool ok = slot < hi;
-      const int page = ok ? page_of(slot / kPage) : 0;
-      const char* src = L.pages + (size_t)page * L.page_bytes +
-                        (size_t)(ok ? slot % kPage : 0) * ROW + (size_t)which * kPage * ROW + j * 16;
+      const int page = ok ? pg[k >> 1] : 0;
+      const char* src = L.pages + (size_t)page * L.page_bytes + (size_t)(ok ? slot % kPage : 0) * ROW +
+                        (size_t)which * kPage * ROW + j * 16;
       cp_async16_zfill(dst + pa_swz(rr, j), src, ok);
+    }
+  };
+  // the page ids of slot tile jt of a head (those holding slots below hi)
+  auto tile_pages = [&](const int* pt, int jt, int hi, int* pg) {
+#pragma unroll
+    for (int q = 0; q < kPaSlots / kPage; ++q) {
+      const int p = jt * (kPaSlots / kPage) + q;
+      pg[q] = p * kPage < hi ? pt[p] : 0;
     }
   };
   auto ptab_of = [&](const Item& w) {
@@ -333,11 +349,11 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
   // see. Copy groups, oldest first: Q (+ carry), K0, V0, then per
   // tile K(j + 1), V(j + 1).
   auto issue_kv0 = [&](const Item& w) {
-    const int* pt = ptab_of(w);
-    auto page_of = [&](int p) { return pt[p]; };
-    load_tile_with(page_of, 0, 0, min(kPaSlots, w.len_final));
+    int pg[kPaSlots / kPage];
+    tile_pages(ptab_of(w), 0, min(kPaSlots, w.len_final), pg);
+    load_tile_pg(pg, 0, 0, min(kPaSlots, w.len_final));
     cp_async_commit();
-    load_tile_with(page_of, 1, 0, min(kPaSlots, w.len_final));
+    load_tile_pg(pg, 1, 0, min(kPaSlots, w.len_final));
     cp_async_commit();
   };
   // an item's carried sums, into copy `par` of the carry buffer (requested with
@@ -411,8 +427,6 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
     // previous item's carry in its epilogue
     cp_async_wait<2>();
     const float* carry = reinterpret_cast<const float*>(smem + kPaCarry + (it & 1) * kPaCarryBytes);
-    auto page_of = [&](int p) { return ptab[p]; };
-    auto load_tile = [&](int which, int jt, int hi) { load_tile_with(page_of, which, jt, hi); };
 
     // ---- per-token decisions, omega, slot counts and 1 / z of the chunk up to
     // the tile end. z after token i is the omega sum of i's segment so far: from
@@ -500,6 +514,10 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
     // so "all but the newest group" always means the tile needed next.
     float m = -INFINITY, l = 0.f;  // l: this thread's half of the row sum
     for (int jt = 0; jt < ntiles; ++jt) {
+      // the next tile's page ids, requested now so that its copies need not
+      // wait for them
+      int pgn[kPaSlots / kPage];
+      tile_pages(ptab, jt + 1, jt + 1 < ntiles ? vis_hi : 0, pgn);
       cp_async_wait<1>();  // Q and K(jt) have landed (this thread's copies)
       fence_async_smem();
       __syncthreads();
@@ -516,7 +534,7 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
       }
       wait_bar(0);  // S is in TMEM and the K buffer is free
       tc_fence_after();
-      if (jt + 1 < ntiles) load_tile(0, jt + 1, vis_hi);
+      if (jt + 1 < ntiles) load_tile_pg(pgn, 0, jt + 1, vis_hi);
       cp_async_commit();
       // ---- online softmax: this thread's half of the row. The running maximum m
       // moves only when a tile's row maximum exceeds it by more than 8 (P then
@@ -610,7 +628,7 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
       // P V done: O holds this tile, S (P) and the V buffer are free
       wait_bar(1);
       tc_fence_after();
-      if (jt + 1 < ntiles) load_tile(1, jt + 1, vis_hi);
+      if (jt + 1 < ntiles) load_tile_pg(pgn, 1, jt + 1, vis_hi);
       cp_async_commit();
     }
     cp_async_wait<0>();
