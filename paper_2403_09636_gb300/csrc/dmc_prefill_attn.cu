@@ -320,17 +320,19 @@ __global__ void __launch_bounds__(kPaThreads, 2) dmc_prefill_attn_kernel(const P
   // compile-time index.
   static_assert(kPaThreads == 256 && kPaSlots == 4 * kPage, "row k of a thread lies in page k / 2");
   auto load_tile_pg = [&](const int* pg, int which, int jt, int hi) {
-    const uint32_t dst = smem_u32(smem + (which ? kPaV : kPaK));
-    const int j = tid & 15;
+    // row r + 16 k: page k / 2, row r + 16 (k & 1) of it, at pa_swz(r, j) + 16 k
+    // rows of 128 bytes in shared memory (r + 16 k and r have the same swizzle)
+    const int r = tid >> 4, j = tid & 15;
+    const uint32_t dst = smem_u32(smem + (which ? kPaV : kPaK)) + pa_swz(r, j);
+    const size_t off = (size_t)r * ROW + (size_t)which * kPage * ROW + j * 16;
+    const int lim = hi - jt * kPaSlots - r;  // row r + 16 k is a slot below hi iff 16 k < lim
+    const char* pb[kPaSlots / kPage];
+#pragma unroll
+    for (int q = 0; q < kPaSlots / kPage; ++q) pb[q] = L.pages + (size_t)pg[q] * L.page_bytes + off;
 #pragma unroll
     for (int k = 0; k < kPaSlots * 16 / kPaThreads; ++k) {
-      const int rr = (tid >> 4) + 16 * k;
-      const int slot = jt * kPaSlots + rr;
-      const bool ok = slot < hi;
-      const int page = ok ? pg[k >> 1] : 0;
-      const char* src = L.pages + (size_t)page * L.page_bytes + (size_t)(ok ? slot % kPage : 0) * ROW +
-                        (size_t)which * kPage * ROW + j * 16;
-      cp_async16_zfill(dst + pa_swz(rr, j), src, ok);
+      const bool ok = 16 * k < lim;
+      cp_async16_zfill(dst + k * 16 * 128, ok ? pb[k >> 1] + (k & 1) * 16 * ROW : L.pages, ok);
     }
   };
   // the page ids of slot tile jt of a head (those holding slots below hi)
