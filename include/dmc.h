@@ -190,10 +190,10 @@ dmc_status dmc_decode_step_layers(dmc_cache_t cache, int32_t first_layer, int32_
  * loading the library holds until the process exits. One launch needs
  *   2 * grid * 8 states of head_dim + 4 floats   (CUDA-core kernel: MHA, fp32,
  *                                                 groups above 8), or
- *   2 * grid * 6 * G states of head_dim + 2 floats (tensor-core kernel: bf16
+ *   2 * grid * 4 * G states of head_dim + 2 floats (tensor-core kernel: bf16
  *                                                 groups of 2 to 8 queries),
  * grid being the cache's decode grid (at most one or two blocks per SM). Every
- * MHA grid fits; a tensor-core grid of group 8 and head_dim 128 fits up to 168
+ * MHA grid fits; a tensor-core grid of group 8 and head_dim 128 fits up to 252
  * blocks (a GB300 runs 152). A grid that does not fit is cut to the blocks
  * that do: the work split follows the grid, so the results then differ from
  * dmc_decode_step's only by the rounding of the split-K sums; when it fits,

@@ -14,12 +14,12 @@ constexpr int kPrefillChunk = 128;     // prompt tokens per prefill block
 constexpr int kMaxVirtualHeads = 16384;
 constexpr int kMaxWindow = 32;         // longest window of the window-grouping approximation
 constexpr int kDecodeWarpsPerBlock = 8;  // worker warps per block, CUDA-core decode kernel
-constexpr int kGqaWarpsPerBlock = 6;     // worker warps per block, tensor-core decode kernel
+constexpr int kGqaWarpsPerBlock = 4;     // worker warps per block, tensor-core decode kernel
 // split-K partial states per layer a cache holds for the decode kernels: two
 // per worker warp of the largest grid (CUDA-core kernel: 512 blocks x 8 warps;
-// tensor-core kernel: 256 blocks x 6 warps, times the group's queries)
+// tensor-core kernel: 256 blocks x 4 warps, times the group's queries)
 constexpr int kMaxWorkerStates = 8192;
-constexpr int kGqaWorkerStates = 3072;
+constexpr int kGqaWorkerStates = 2048;
 
 // Device-side view of one cache. Passed by value to every kernel.
 struct Layout {
