@@ -188,7 +188,7 @@ dmc_status dmc_decode_step_layers(dmc_cache_t cache, int32_t first_layer, int32_
  * The scratch is the split-K partial softmax states of one launch, kept in a
  * file-scope __device__ array of 8 MiB (2,097,152 floats) that every GPU
  * loading the library holds until the process exits. One launch needs
- *   2 * grid * 8 states of head_dim + 4 floats   (CUDA-core kernel: MHA, fp32,
+ *   2 * grid * 6 states of head_dim + 4 floats   (CUDA-core kernel: MHA, fp32,
  *                                                 groups above 8), or
  *   2 * grid * 4 * G states of head_dim + 2 floats (tensor-core kernel: bf16
  *                                                 groups of 2 to 8 queries),

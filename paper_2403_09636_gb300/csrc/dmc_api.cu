@@ -28,7 +28,7 @@ cudaError_t gqa_setup(const Layout& L, DecodePlan* plan);
 cudaError_t gqa_launch(const Layout& L, int layer0, int nlayers, const DecodePlan& plan, bool pdl, const void* q,
                        const void* k, const void* v, void* out, cudaStream_t stream);
 // Split-K partial states a cache's arena holds: two per worker warp of the
-// decode grid (at most 512 blocks x 8 warps), times the group size for the
+// decode grid (at most 512 blocks x 6 warps), times the group size for the
 // tensor-core kernel, which keeps one per query.
 inline size_t partial_states_cap(bool cuda_core, int G) {
   return cuda_core ? (size_t)kMaxWorkerStates : (size_t)kGqaWorkerStates * G;
@@ -361,8 +361,8 @@ dmc_status dmc_decode_step_static_scratch(dmc_cache_t c, int32_t layer, const vo
   e = dmc::decode_static_partials(dev, &scratch, &floats);
   if (e != cudaSuccess) return DMC_ERR_CUDA;
   // One launch writes two partial states per worker warp: of head_dim + 4
-  // floats for the CUDA-core kernel (8 warps per block), and one per query
-  // of the group, of head_dim + 2 floats, for the tensor-core kernel (6 warps
+  // floats for the CUDA-core kernel (6 warps per block), and one per query
+  // of the group, of head_dim + 2 floats, for the tensor-core kernel (4 warps
   // per block). A grid that needs more than the array holds is cut to fit;
   // the work split follows the grid, so results differ from dmc_decode_step's
   // only by the order of the split-K sums.

@@ -43,14 +43,18 @@
 
 namespace dmc {
 
-constexpr int kWarps = kDecodeWarpsPerBlock;  // independent workers per block
-constexpr int kDecodeThreads = kWarps * 32;
-constexpr int kRing = 6;        // quads per warp ring (kRing - 1 in flight)
+// Worker warps per block: a launch over one layer ends with a tail (its last
+// heads finish while other warps idle), which fewer, longer warp ranges make
+// shorter; a launch over several layers pays the tail once, and streams faster
+// with more warps in flight.
+constexpr int kWarpsOne = kDecodeWarpsPerBlock;
+constexpr int kWarpsWalk = kDecodeWalkWarpsPerBlock;
+constexpr int kRing = 5;        // quads per warp ring (kRing - 1 in flight)
 constexpr int kWindow = 64;     // page units per warp window (page id + rows to copy)
 constexpr int kHeadWindow = 32; // heads whose gates a warp holds in its lanes
 constexpr int kMaxDecodeBlocks = 512;
-constexpr int kMaxWorkers = kMaxDecodeBlocks * kWarps;
-static_assert(kMaxWorkers * 2 == 8192, "partials hold two states per worker");
+constexpr int kMaxWorkers = kMaxDecodeBlocks * (kWarpsOne > kWarpsWalk ? kWarpsOne : kWarpsWalk);
+static_assert(kMaxWorkers * 2 <= kMaxWorkerStates, "partials hold two states per worker");
 
 enum : int { kFlagAcc = 1, kFlagNaN = 2 };
 
@@ -77,8 +81,8 @@ struct DecodeGeom {
   static constexpr int WWIN = 2 * kWindow * 4;  // page ids, rows to copy
   static constexpr int WARP_BYTES = WRING + WWIN;
   static constexpr int MISC = 64;
-  static size_t smem_bytes(int nvh) {
-    return (size_t)kWarps * WARP_BYTES + MISC + (size_t)(nvh + 1) * 4;
+  static size_t smem_bytes(int nvh, int warps) {
+    return (size_t)warps * WARP_BYTES + MISC + (size_t)(nvh + 1) * 4;
   }
 };
 
@@ -187,9 +191,10 @@ __device__ __noinline__ void combine_partials(const float* partials, int wf, int
   }
 }
 
-// kWin: the cache uses the window-grouping approximation (L.window > 0)
-template <typename T, int D, bool kWin>
-__global__ void __launch_bounds__(kDecodeThreads, 2)
+// kWin: the cache uses the window-grouping approximation (L.window > 0);
+// NWARP: worker warps per block
+template <typename T, int D, bool kWin, int NWARP>
+__global__ void __launch_bounds__(NWARP * 32, 2)
 dmc_decode_kernel(const DecodeArgs a) {
   using G_ = DecodeGeom<T, D>;
   using CK = Chunk<T>;
@@ -204,7 +209,7 @@ dmc_decode_kernel(const DecodeArgs a) {
   unsigned char* ring = smem + (size_t)warp * G_::WARP_BYTES;
   int* wpid = reinterpret_cast<int*>(ring + G_::WRING);
   int* wrws = wpid + kWindow;
-  int* misc = reinterpret_cast<int*>(smem + (size_t)kWarps * G_::WARP_BYTES);
+  int* misc = reinterpret_cast<int*>(smem + (size_t)NWARP * G_::WARP_BYTES);
   int* U = misc + G_::MISC / 4;
 
   for (int li = 0; li < a.nlayers; ++li) {
@@ -227,8 +232,8 @@ dmc_decode_kernel(const DecodeArgs a) {
   // ---------------------------------------------------------------- prologue
   scan_units(U, misc, ctl, L.lengths + (size_t)layer * 2 * L.NH, L.NH, NVH, Gv);
   const long long Utot = U[NVH];
-  const int NW = gridDim.x * kWarps;
-  const int wid = blockIdx.x * kWarps + warp;
+  const int NW = gridDim.x * NWARP;
+  const int wid = blockIdx.x * NWARP + warp;
   const int u0 = (int)range_start(wid, Utot, NW);
   const int u1 = (int)range_start(wid + 1, Utot, NW);
   const int grp = lane >> 3, l8 = lane & 7;
@@ -698,7 +703,7 @@ dmc_decode_kernel(const DecodeArgs a) {
     // last block of the launch: every owner has finished
     if (Gv > 1) {
       __threadfence();
-      for (int bh = tid; bh < L.NH; bh += kDecodeThreads) {
+      for (int bh = tid; bh < L.NH; bh += NWARP * 32) {
         const int at = pending_at[bh];
         if (at < 0) continue;
         char* dst = L.pages + (size_t)(at / kPage) * L.page_bytes + (size_t)(at % kPage) * ROW;
@@ -722,33 +727,42 @@ dmc_decode_kernel(const DecodeArgs a) {
   }  // layers
 }
 
+// Shared memory and blocks per SM of one warp count (both window variants).
+template <typename T, int D, int NWARP>
+static cudaError_t setup_warps(int nvh, int optin, size_t* smem, int* occ) {
+  *smem = DecodeGeom<T, D>::smem_bytes(nvh, NWARP);
+  if (*smem > (size_t)optin) return cudaErrorInvalidConfiguration;
+  cudaError_t e = cudaFuncSetAttribute(dmc_decode_kernel<T, D, false, NWARP>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)*smem);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(dmc_decode_kernel<T, D, true, NWARP>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)*smem);
+  int o = 0, ow = 0;
+  if (e == cudaSuccess)
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o, dmc_decode_kernel<T, D, false, NWARP>, NWARP * 32,
+                                                      *smem);
+  if (e == cudaSuccess)
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&ow, dmc_decode_kernel<T, D, true, NWARP>, NWARP * 32,
+                                                      *smem);
+  if (e != cudaSuccess) return e;
+  *occ = min(o, ow);
+  return *occ < 1 ? cudaErrorInvalidConfiguration : cudaSuccess;
+}
+
 template <typename T, int D>
 static cudaError_t setup_decode(int nvh, DecodePlan* plan) {
-  using G_ = DecodeGeom<T, D>;
   int dev = 0, sms = 0, optin = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
   if (e != cudaSuccess) return e;
   plan->stages = kRing;
-  plan->smem = G_::smem_bytes(nvh);
-  if (plan->smem > (size_t)optin) return cudaErrorInvalidConfiguration;
-  e = cudaFuncSetAttribute(dmc_decode_kernel<T, D, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                           (int)plan->smem);
-  if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(dmc_decode_kernel<T, D, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)plan->smem);
-  if (e != cudaSuccess) return e;
   int occ = 0, occw = 0;
-  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, dmc_decode_kernel<T, D, false>, kDecodeThreads,
-                                                    plan->smem);
-  if (e == cudaSuccess)
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occw, dmc_decode_kernel<T, D, true>,
-                                                      kDecodeThreads, plan->smem);
-  occ = min(occ, occw);
+  e = setup_warps<T, D, kWarpsOne>(nvh, optin, &plan->smem, &occ);
+  if (e == cudaSuccess) e = setup_warps<T, D, kWarpsWalk>(nvh, optin, &plan->smem_walk, &occw);
   if (e != cudaSuccess) return e;
-  if (occ < 1) return cudaErrorInvalidConfiguration;
   plan->grid = min(sms * occ, kMaxDecodeBlocks);
+  plan->grid_walk = min(sms * occw, kMaxDecodeBlocks);
   return cudaSuccess;
 }
 
@@ -759,30 +773,37 @@ cudaError_t decode_setup(const Layout& L, int Gv, DecodePlan* plan) {
   if (L.esize == 4 && L.D == 128) e = setup_decode<float, 128>(nvh, plan);
   if (L.esize == 2 && L.D == 64) e = setup_decode<__nv_bfloat16, 64>(nvh, plan);
   if (L.esize == 2 && L.D == 128) e = setup_decode<__nv_bfloat16, 128>(nvh, plan);
+  if (e != cudaSuccess) return e;
   // no more warps than the most units a layer can have
   const long long max_units = (long long)nvh * (L.MPH + 1);
-  const long long max_blocks = (max_units + kWarps - 1) / kWarps;
-  if (e == cudaSuccess && max_blocks < plan->grid) plan->grid = (int)max_blocks;
-  plan->partial_states = 2 * plan->grid * kWarps;
-  if (e == cudaSuccess && plan->partial_states > L.partial_cap) e = cudaErrorInvalidConfiguration;
-  return e;
+  plan->grid = (int)std::min<long long>(plan->grid, (max_units + kWarpsOne - 1) / kWarpsOne);
+  plan->grid_walk = (int)std::min<long long>(plan->grid_walk, (max_units + kWarpsWalk - 1) / kWarpsWalk);
+  plan->partial_states = 2 * max(plan->grid * kWarpsOne, plan->grid_walk * kWarpsWalk);
+  if (plan->partial_states > L.partial_cap) return cudaErrorInvalidConfiguration;
+  return cudaSuccess;
 }
 
-template <typename T, int D>
-static cudaError_t launch_decode(const DecodeArgs& a, const DecodePlan& plan, bool pdl,
-                                 cudaStream_t stream) {
+template <typename T, int D, int NWARP>
+static cudaError_t launch_warps(const DecodeArgs& a, int grid, size_t smem, bool pdl, cudaStream_t stream) {
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(plan.grid);
-  cfg.blockDim = dim3(kDecodeThreads);
-  cfg.dynamicSmemBytes = plan.smem;
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(NWARP * 32);
+  cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = pdl ? 1 : 0;
-  if (a.lay.window > 0) return cudaLaunchKernelEx(&cfg, dmc_decode_kernel<T, D, true>, a);
-  return cudaLaunchKernelEx(&cfg, dmc_decode_kernel<T, D, false>, a);
+  if (a.lay.window > 0) return cudaLaunchKernelEx(&cfg, dmc_decode_kernel<T, D, true, NWARP>, a);
+  return cudaLaunchKernelEx(&cfg, dmc_decode_kernel<T, D, false, NWARP>, a);
+}
+
+template <typename T, int D>
+static cudaError_t launch_decode(const DecodeArgs& a, const DecodePlan& plan, bool pdl,
+                                 cudaStream_t stream) {
+  if (a.nlayers > 1) return launch_warps<T, D, kWarpsWalk>(a, plan.grid_walk, plan.smem_walk, pdl, stream);
+  return launch_warps<T, D, kWarpsOne>(a, plan.grid, plan.smem, pdl, stream);
 }
 
 cudaError_t decode_launch(const Layout& L, int layer0, int nlayers, int Gv, const DecodePlan& plan,
@@ -813,7 +834,7 @@ cudaError_t decode_launch(const Layout& L, int layer0, int nlayers, int Gv, cons
 // of one launch, 8 MiB. That holds two states of head_dim + 4 floats for each
 // of the MHA kernel's 4096 worker warps at most, and the tensor-core kernel's
 // two states per query of a group of 8 (head_dim + 2 floats each) for up to
-// 168 blocks of 6 warps (a GB300 runs 152). Every GPU that loads the library
+// 252 blocks of 4 warps (a GB300 runs 152). Every GPU that loads the library
 // holds it until exit.
 constexpr size_t kStaticPartialFloats = (size_t)2 << 20;
 static_assert(kStaticPartialFloats >= (size_t)2 * kMaxWorkers * kPartialStride<128>,

@@ -639,6 +639,8 @@ static cudaError_t setup_gqa(const Layout& L, DecodePlan* plan) {
   const long long max_blocks = (max_units + kGWarps - 1) / kGWarps;
   if (max_blocks < plan->grid) plan->grid = (int)max_blocks;
   plan->partial_states = 2 * plan->grid * kGWarps * L.G;
+  plan->grid_walk = plan->grid;  // one launch shape whatever the layers
+  plan->smem_walk = plan->smem;
   if (plan->partial_states > L.partial_cap) return cudaErrorInvalidConfiguration;
   return cudaSuccess;
 }

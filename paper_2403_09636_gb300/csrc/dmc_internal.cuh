@@ -13,8 +13,9 @@ constexpr int kPage = 32;              // slots per page (the paper's page size)
 constexpr int kPrefillChunk = 128;     // prompt tokens per prefill block
 constexpr int kMaxVirtualHeads = 16384;
 constexpr int kMaxWindow = 32;         // longest window of the window-grouping approximation
-constexpr int kDecodeWarpsPerBlock = 8;  // worker warps per block, CUDA-core decode kernel
-constexpr int kGqaWarpsPerBlock = 4;     // worker warps per block, tensor-core decode kernel
+constexpr int kDecodeWarpsPerBlock = 6;      // worker warps per block, CUDA-core decode kernel
+constexpr int kDecodeWalkWarpsPerBlock = 8;  // the same, for a launch over several layers
+constexpr int kGqaWarpsPerBlock = 4;         // worker warps per block, tensor-core decode kernel
 // split-K partial states per layer a cache holds for the decode kernels: two
 // per worker warp of the largest grid (CUDA-core kernel: 512 blocks x 8 warps;
 // tensor-core kernel: 256 blocks x 4 warps, times the group's queries)
@@ -60,10 +61,12 @@ __host__ __device__ inline int ceil_div(int a, int b) { return (a + b - 1) / b; 
 
 // Launch shape of the decode kernel for one cache, fixed at create time.
 struct DecodePlan {
-  int grid;            // blocks
+  int grid;            // blocks of a launch over one layer
   int stages;          // shared-memory ring depth (quads per warp)
   int partial_states;  // split-K partial states one launch may write
   size_t smem;         // dynamic shared memory per block
+  int grid_walk;       // blocks and shared memory of a CUDA-core launch over several
+  size_t smem_walk;    // layers (its own warp count); the tensor-core kernel uses grid, smem
 };
 
 // ---------------------------------------------------------------- dtype helpers
