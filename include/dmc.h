@@ -165,9 +165,13 @@ dmc_status dmc_decode_step(dmc_cache_t cache, int32_t layer, const void* q_dev,
 /* dmc_decode_step for the layers [first_layer, first_layer + num_layers) in
  * one launch, when the inputs of all of them are ready (the step of each layer
  * reads only that layer's cache and inputs, Algorithm 1 and Eq. attn-softmax
- * per KV head, so the layers are independent). Same result for every layer as
- * calling dmc_decode_step on the layers in order; what it saves is one launch
- * and one kernel start-up and tail per layer, which dominate small caches.
+ * per KV head, so the layers are independent). Same slots and lengths for
+ * every layer as calling dmc_decode_step on the layers in order, and the same
+ * outputs up to the order of the split-K sums: the CUDA-core kernel runs more
+ * warps per block over several layers than over one, so a head may be split
+ * over other warps (outputs are bit-identical when neither grid splits a head,
+ * and always for the tensor-core kernel). What it saves is one launch and one
+ * kernel start-up and tail per layer, which dominate small caches.
  *   q_dev:   [num_layers, batch, num_q_heads, head_dim]
  *   k_dev, v_dev: [num_layers, batch, num_kv_heads, head_dim]
  *   out_dev: [num_layers, batch, num_q_heads, head_dim] (written)

@@ -460,11 +460,25 @@ dmc_decode_kernel(const DecodeArgs a) {
             rz += __shfl_xor_sync(0xffffffffu, rz, off);
           }
         }
-        if (grp == 0) {
+        // When this warp has just streamed the head's last page (unit u - 1),
+        // its last quad holds the old last row in the ring, in the lanes of row
+        // group (len_old - 1) % 4, and the issue window may still hold that
+        // page's id: that group then applies the update without a round trip
+        // for either.
+        const bool ring_row = !kWin && accum && k > 0 && j > 0;
+        const int og = ring_row ? ((len_old - 1) & 3) : 0;
+        const unsigned gmask = 0xffu << (8 * og);
+        if (grp == og) {
         // Algorithm 1 on the new token, in fp32, result rounded to the cache dtype.
-        const int* pt_row = ptab + (size_t)bh * L.MPH;
         int tgt = -1;
-        if (accum || len_old % kPage != 0) tgt = pt_row[(len_old - 1) / kPage];
+        if (accum || len_old % kPage != 0) {
+          const int up = u - 1;
+          tgt = (k > 0 && j > 0 && up >= pb && up - pb < kWindow)
+                    ? wpid[up - pb]
+                    : ptab[(size_t)bh * L.MPH + (len_old - 1) / kPage];
+        }
+        const unsigned char* rrow =
+            ring + (size_t)((cslot == 0 ? kRing : cslot) - 1) * G_::WSLOT + lane * 16;
         float zold = 0.f, znew = omega;
         const char* orow = nullptr;
         // window grouping: the slot is the mean of the segment's last W
@@ -502,8 +516,13 @@ dmc_decode_kernel(const DecodeArgs a) {
             }
           } else if (accum) {
             float ko[EPC], vo[EPC];
-            CK::unpack(*reinterpret_cast<const uint4*>(orow + c * 128 + l8 * 16), ko);
-            CK::unpack(*reinterpret_cast<const uint4*>(orow + (size_t)kPage * ROW + c * 128 + l8 * 16), vo);
+            if (ring_row) {
+              CK::unpack(*reinterpret_cast<const uint4*>(rrow + c * 512), ko);
+              CK::unpack(*reinterpret_cast<const uint4*>(rrow + (NCH + c) * 512), vo);
+            } else {
+              CK::unpack(*reinterpret_cast<const uint4*>(orow + c * 128 + l8 * 16), ko);
+              CK::unpack(*reinterpret_cast<const uint4*>(orow + (size_t)kPage * ROW + c * 128 + l8 * 16), vo);
+            }
 #pragma unroll
             for (int e = 0; e < EPC; ++e) {
               kn[e] = (ko[e] * zold + kin[e] * omega) / znew;
@@ -536,7 +555,7 @@ dmc_decode_kernel(const DecodeArgs a) {
                 ptab[(size_t)bh * L.MPH + slot / kPage] = page;
               }
             }
-            page = __shfl_sync(0xffu, page, 0, 8);
+            page = __shfl_sync(gmask, page, 0, 8);
           }
           ok = ok && page >= 0;
           // With grouped queries the other virtual heads of this KV head may
@@ -567,9 +586,9 @@ dmc_decode_kernel(const DecodeArgs a) {
             if (flags & kFlagNaN) atomicOr(L.error, DMC_FAULT_NAN_GATE);
           }
         }
-        s += __shfl_xor_sync(0xffu, s, 1);
-        s += __shfl_xor_sync(0xffu, s, 2);
-        s += __shfl_xor_sync(0xffu, s, 4);
+        s += __shfl_xor_sync(gmask, s, 1);
+        s += __shfl_xor_sync(gmask, s, 2);
+        s += __shfl_xor_sync(gmask, s, 4);
         const float mn = fmaxf(m, s);
         const float corr = exp2f(m - mn);
         const float p = exp2f(s - mn);
@@ -759,11 +778,14 @@ static cudaError_t setup_decode(int nvh, DecodePlan* plan) {
   plan->stages = kRing;
   int occ = 0, occw = 0;
   e = setup_warps<T, D, kWarpsOne>(nvh, optin, &plan->smem, &occ);
-  if (e == cudaSuccess) e = setup_warps<T, D, kWarpsWalk>(nvh, optin, &plan->smem_walk, &occw);
   if (e != cudaSuccess) return e;
   plan->grid = min(sms * occ, kMaxDecodeBlocks);
-  plan->grid_walk = min(sms * occw, kMaxDecodeBlocks);
-  return cudaSuccess;
+  // a launch over several layers takes the one-layer shape when its own does
+  // not fit (wide rows with many heads)
+  e = setup_warps<T, D, kWarpsWalk>(nvh, optin, &plan->smem_walk, &occw);
+  plan->grid_walk = e == cudaSuccess ? min(sms * occw, kMaxDecodeBlocks) : 0;
+  if (e == cudaErrorInvalidConfiguration) e = cudaSuccess;
+  return e;
 }
 
 cudaError_t decode_setup(const Layout& L, int Gv, DecodePlan* plan) {
@@ -802,7 +824,8 @@ static cudaError_t launch_warps(const DecodeArgs& a, int grid, size_t smem, bool
 template <typename T, int D>
 static cudaError_t launch_decode(const DecodeArgs& a, const DecodePlan& plan, bool pdl,
                                  cudaStream_t stream) {
-  if (a.nlayers > 1) return launch_warps<T, D, kWarpsWalk>(a, plan.grid_walk, plan.smem_walk, pdl, stream);
+  if (a.nlayers > 1 && plan.grid_walk > 0)
+    return launch_warps<T, D, kWarpsWalk>(a, plan.grid_walk, plan.smem_walk, pdl, stream);
   return launch_warps<T, D, kWarpsOne>(a, plan.grid, plan.smem, pdl, stream);
 }
 

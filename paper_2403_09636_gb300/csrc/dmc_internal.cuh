@@ -66,7 +66,8 @@ struct DecodePlan {
   int partial_states;  // split-K partial states one launch may write
   size_t smem;         // dynamic shared memory per block
   int grid_walk;       // blocks and shared memory of a CUDA-core launch over several
-  size_t smem_walk;    // layers (its own warp count); the tensor-core kernel uses grid, smem
+  size_t smem_walk;    // layers (its own warp count; grid_walk 0: the one-layer shape);
+                       // the tensor-core kernel uses grid, smem
 };
 
 // ---------------------------------------------------------------- dtype helpers
