@@ -362,14 +362,32 @@ __global__ void __launch_bounds__(kGThreads, 1) dmc_decode_gqa_kernel(const GqaA
         // Algorithm 1 on the KV head's new token, once for the group: lanes
         // 0..CPR-1 build the key row, lanes CPR..2*CPR-1 the value row, 8
         // dims each, in fp32, rounded to bf16.
+        const bool is_v = lane >= CPR;
+        const int c = is_v ? lane - CPR : lane;
+        const bool act = lane < 2 * CPR;
+        // When this warp has just streamed the head's last page (unit u - 1),
+        // the old last row is in the tile it consumed last: read it before
+        // the issue below reuses that ring slot. The issue window may still
+        // hold that page's id.
+        const bool ring_row = !kWin && accum && k > 0 && j > 0;
+        uint4 oraw = make_uint4(0, 0, 0, 0);
+        if (ring_row && act) {
+          const int ps = (cslot == 0 ? kGRing : cslot) - 1;
+          oraw = *reinterpret_cast<const uint4*>(smem + (ring_s - smem_u32(smem)) + ps * G_::TILE +
+                                                 (is_v ? kTile * ROW : 0) + swz((len_old - 1) % kTile, c, ROW));
+        }
         issue_next();
         cp_async_wait<kGRing - 1>();
         __syncwarp();  // the reserved tile's slot is free
         const uint32_t tile = ring_s + cslot * G_::TILE;
         cslot = (cslot + 1 == kGRing) ? 0 : cslot + 1;
-        const int* pt_row = ptab + (size_t)vh * L.MPH;
         int tgt = -1;
-        if (accum || len_old % kPage != 0) tgt = pt_row[(len_old - 1) / kPage];
+        if (accum || len_old % kPage != 0) {
+          const int up = u - 1;
+          tgt = (k > 0 && j > 0 && up >= pb && up - pb < kGWindow)
+                    ? wpid[up - pb]
+                    : ptab[(size_t)vh * L.MPH + (len_old - 1) / kPage];
+        }
         // window grouping: the slot is the mean of the segment's last W tokens,
         // the W - 1 before this one being in the head's ring
         const int W = kWin ? L.window : 0;
@@ -390,9 +408,6 @@ __global__ void __launch_bounds__(kGThreads, 1) dmc_decode_gqa_kernel(const GqaA
           zold = L.z[(size_t)tgt * kPage + (len_old - 1) % kPage];
           znew = zold + omega;
         }
-        const bool is_v = lane >= CPR;
-        const int c = is_v ? lane - CPR : lane;
-        const bool act = lane < 2 * CPR;
         uint4 nrow = make_uint4(0, 0, 0, 0);
         if (act) {
           float in[8], nw[8];
@@ -416,10 +431,14 @@ __global__ void __launch_bounds__(kGThreads, 1) dmc_decode_gqa_kernel(const GqaA
             char* re = L.ring + ((size_t)layer * NH + vh) * W * 2 * ROW + (size_t)(n_old % Wm) * 2 * ROW;
             *reinterpret_cast<uint4*>(re + (is_v ? ROW : 0) + c * 16) = CK::pack(in);
           } else if (accum) {
-            const char* orow = L.pages + (size_t)tgt * L.page_bytes +
-                               (size_t)(is_v ? kPage : 0) * ROW + (size_t)((len_old - 1) % kPage) * ROW;
             float old[8];
-            CK::unpack(*reinterpret_cast<const uint4*>(orow + c * 16), old);
+            if (ring_row) {
+              CK::unpack(oraw, old);
+            } else {
+              const char* orow = L.pages + (size_t)tgt * L.page_bytes +
+                                 (size_t)(is_v ? kPage : 0) * ROW + (size_t)((len_old - 1) % kPage) * ROW;
+              CK::unpack(*reinterpret_cast<const uint4*>(orow + c * 16), old);
+            }
 #pragma unroll
             for (int e = 0; e < 8; ++e) nw[e] = (old[e] * zold + in[e] * omega) / znew;
           } else {
