@@ -54,6 +54,22 @@ def test_f32_head_dim_128(cuda_dev):
     _check(H.Run(wl, cuda_dev, H.all_samples(wl)))
 
 
+@pytest.mark.parametrize("wl", [
+    # fp32 MHA at d 128 (one block per SM: 912 warps) over ~2,800 units, and
+    # fp32 grouped queries at d 64 (two virtual heads per KV head on the
+    # CUDA-core kernel, 1,824 warps) over ~5,000: ranges of several units, so
+    # an owner unit usually follows its head's last page in the same warp,
+    # which then takes the old last row from its own ring. CR 1.25-2 keeps
+    # merges frequent.
+    S.Workload("f32_d128_dense", 1, 6, 8, 8, 128, "f32", (2600, 3000), 8, ("choice", (1.25, 2.0)),
+               1.0, seed=5),
+    S.Workload("f32_d64_g2_dense", 1, 6, 16, 8, 64, "f32", (2600, 3000), 8, ("choice", (1.25, 2.0)),
+               1.0, seed=6),
+], ids=lambda w: w.name)
+def test_f32_ranges_of_several_units(cuda_dev, wl):
+    _check(H.Run(wl, cuda_dev, H.all_samples(wl)))
+
+
 def test_gqa_virtual_heads_read_the_old_last_slot(cuda_dev):
     """Every query of a group merges the new token into the same old last
     slot; the group's one writer must not let another query see the merged

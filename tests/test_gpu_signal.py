@@ -17,7 +17,8 @@ Each case checks, per head:
     query ignored, the 1/sqrt(d_h) scale left out, one 32-slot page dropped;
     tests/mutants.py), so that each mistake would fail the test.
 Covered: the MHA CUDA-core kernel (d 128 and 64, dense and sparse unit
-ranges), the grouped-query mma.sync kernel (G = 2, 4, 8) and the prompt
+ranges), the grouped-query mma.sync kernel (G = 2, 4, 8; d 128 and 64, dense
+and sparse unit ranges) and the prompt
 attention tcgen05 kernel (G = 1, 2, 4, 8). The observed errors are printed.
 """
 import numpy as np
@@ -51,6 +52,11 @@ DECODE = [
     _wl("sig_gqa_g4_d64", 1, 4, 8, 2, 64, (20, 2600), 16, ("choice", (1.0, 2.0)), 306),
     # 32 long grouped heads: more units than the tensor-core kernel's warps
     _wl("sig_gqa_g8_dense", 1, 8, 32, 4, 128, (1500, 3000), 12, ("fixed", 1.0), 307),
+    # several units per warp at d 64, on the MHA kernel and the tensor-core
+    # kernel, with frequent merges (an owner unit after its head's last page in
+    # the same warp takes the old last row from that warp's ring)
+    _wl("sig_mha_d64_dense", 1, 12, 8, 8, 64, (2000, 3000), 10, ("choice", (1.25, 2.0)), 308),
+    _wl("sig_gqa_g4_d64_dense", 1, 8, 32, 8, 64, (2000, 3000), 10, ("choice", (1.25, 2.0)), 309),
 ]
 
 
